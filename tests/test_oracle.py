@@ -1,0 +1,244 @@
+"""Pins for the CPU oracle: what the paper and the mathematics fix, not the
+oracle's own code.  CPU only."""
+import math
+import os
+
+import numpy as np
+import pytest
+from scipy.special import expit
+
+from oracle import bp_oracle as O
+from paper_1801_01554_gb300 import synth
+
+GOLDEN = os.path.join(os.path.dirname(__file__), "golden")
+
+
+def _golden(name):
+    out = {}
+    with open(os.path.join(GOLDEN, name)) as f:
+        for line in f:
+            line = line.split("#", 1)[0].strip()
+            if line:
+                k, *v = line.split()
+                out[k] = [float(x) for x in v]
+    return out
+
+
+# ------------------------------------------------------------------ counting
+def test_connection_count_matches_paper():
+    g = _golden("nettalk_counts.txt")
+    sizes = tuple(int(x) for x in g["sizes"])
+    assert O.connections(sizes) == int(g["connections"][0])
+
+
+def test_flop_factor_matches_paper():
+    g = _golden("nettalk_counts.txt")
+    sizes = tuple(int(x) for x in g["sizes"])
+    f = O.flops_per_connection(sizes)
+    assert round(f, 2) == g["flop_factor"][0]
+    # 901 MCPS x 4.23 = 3.8 GFLOPS (Section 7.2)
+    assert round(g["mcps"][0] * f / 1000.0, 1) == g["gflops"][0]
+    # the per-pattern cycle counts of Section 6.1 give the same factor
+    assert O.flops_per_pattern(sizes) == pytest.approx(f * O.connections(sizes), rel=1e-12)
+
+
+# ------------------------------------------------------------------ sigmoid
+def test_sigmoid_against_library_and_symmetry():
+    x = np.linspace(-40, 40, 2001)
+    np.testing.assert_allclose(O.sigmoid(x), expit(x), rtol=1e-14, atol=1e-300)
+    assert O.sigmoid(0.0) == 0.5
+    np.testing.assert_allclose(O.sigmoid(-x), 1.0 - O.sigmoid(x), atol=1e-15)
+
+
+def test_sigmoid_derivative_identity():
+    # sigma'(x) = sigma(x)(1 - sigma(x)), against central differences of sigma
+    x = np.linspace(-8, 8, 161)
+    h = 1e-5
+    fd = (O.sigmoid(x + h) - O.sigmoid(x - h)) / (2 * h)
+    s = O.sigmoid(x)
+    np.testing.assert_allclose(s * (1 - s), fd, rtol=1e-7, atol=1e-10)
+
+
+# ------------------------------------------------------------------ gradients
+def _half_sse(sizes, theta, X, T):
+    Ws, bs = O.unpack(sizes, theta)
+    return 0.5 * O.sse(O.forward(Ws, bs, X)[-1], T)
+
+
+def fd_relative_error(sizes, n_pat=5, seed=0, h=1e-6):
+    """max |G + dE/dtheta| / max |dE/dtheta| over every weight and bias, with
+    E = SSE/2 and dE/dtheta from central differences."""
+    rng = np.random.default_rng(seed)
+    theta = rng.uniform(-1.0, 1.0, O.connections(sizes))
+    X = rng.standard_normal((n_pat, sizes[0]))
+    T = (rng.random((n_pat, sizes[-1])) < 0.5).astype(float)
+    st = O.State(sizes, theta, lr=0.0, momentum=0.0)
+    _, _, G, _ = O.step_quantities(st, X, T)
+    fd = np.empty_like(theta)
+    for k in range(theta.size):
+        tp = theta.copy(); tp[k] += h
+        tm = theta.copy(); tm[k] -= h
+        fd[k] = (_half_sse(sizes, tp, X, T) - _half_sse(sizes, tm, X, T)) / (2 * h)
+    # G is the pooled delta*activation, i.e. minus the gradient of E/2
+    return np.max(np.abs(G + fd)) / np.max(np.abs(fd))
+
+
+@pytest.mark.parametrize("sizes", [(2, 3, 2), (4, 5, 3, 2), (3, 1), (3, 4, 4, 4, 2)])
+def test_gradient_matches_finite_differences(sizes):
+    assert fd_relative_error(sizes) < 1e-6
+
+
+@pytest.mark.parametrize("mistake", ["sign", "no_derivative", "no_bias_grad", "transposed"])
+def test_planted_mistakes_fail_the_finite_difference_pin(monkeypatch, mistake):
+    """A plausible mistake anywhere in the backward pass must break the pin."""
+    if mistake == "sign":
+        monkeypatch.setattr(O, "output_delta", lambda Oo, T: (Oo - T) * Oo * (1 - Oo))
+    elif mistake == "no_derivative":
+        monkeypatch.setattr(O, "hidden_delta", lambda Wn, Dn, A: Dn @ Wn)
+    elif mistake == "no_bias_grad":
+        real = O.gradients
+        monkeypatch.setattr(O, "gradients",
+                            lambda As, Ds: (real(As, Ds)[0], [0 * D.sum(0) for D in Ds]))
+    elif mistake == "transposed":
+        # square hidden layers so that the transposed product still has the right shape
+        monkeypatch.setattr(O, "hidden_delta", lambda Wn, Dn, A: (Dn @ Wn.T) * A * (1 - A))
+    sizes = (3, 4, 4, 4) if mistake == "transposed" else (2, 3, 2)
+    assert fd_relative_error(sizes) > 1e-2
+
+
+def test_pooled_change_is_sum_of_single_pattern_changes():
+    # Section 4.1: the pooled change is the sum of the per-pattern changes
+    sizes = (7, 6, 3)
+    X, T = synth.gaussian_patterns(9, 7, 3, 0.5, seed=3)
+    st = O.State(sizes, synth.init_uniform(sizes, -0.5, 0.5, 3), 0.1, 0.9)
+    _, _, G, e = O.step_quantities(st, X, T)
+    parts = [O.step_quantities(st, X[p:p + 1], T[p:p + 1]) for p in range(9)]
+    np.testing.assert_allclose(G, sum(q[2] for q in parts), rtol=1e-12, atol=1e-15)
+    assert e == pytest.approx(sum(q[3] for q in parts), rel=1e-12)
+
+
+def test_pooled_change_is_order_independent():
+    # Section 4.1: changes may be applied in any order with the same result
+    sizes = (7, 6, 3)
+    X, T = synth.gaussian_patterns(33, 7, 3, 0.3, seed=4)
+    st = O.State(sizes, synth.init_uniform(sizes, -0.5, 0.5, 4), 0.1, 0.9)
+    perm = np.random.default_rng(1).permutation(33)
+    G1 = O.step_quantities(st, X, T)[2]
+    G2 = O.step_quantities(st, X[perm], T[perm])[2]
+    np.testing.assert_allclose(G1, G2, rtol=1e-12, atol=1e-14)
+
+
+def test_sse_is_plain_sum_of_squares():
+    Oo = np.full((5, 4), 0.5)
+    T = np.ones((5, 4))
+    assert O.sse(Oo, T) == 5 * 4 * 0.25
+
+
+# ------------------------------------------------------------------ update
+def test_zero_learning_rate_leaves_weights_unchanged():
+    sizes = (4, 3, 2)
+    X, T = synth.gaussian_patterns(6, 4, 2, 0.5, seed=5)
+    th = synth.init_uniform(sizes, -0.5, 0.5, 5)
+    for m in (0.0, 0.9):
+        st = O.State(sizes, th, lr=0.0, momentum=m)
+        for _ in range(3):
+            O.train_batch(st, X, T)
+        np.testing.assert_array_equal(st.theta, th)
+        assert not st.G.any()
+
+
+def test_momentum_closed_form_under_constant_change():
+    # with the same pooled change g every time, V_k = lr g (1 - m^k)/(1 - m)
+    # and W_k = W_0 + lr g sum_{j=1..k} (1 - m^j)/(1 - m)
+    rng = np.random.default_rng(7)
+    w0 = rng.standard_normal(10)
+    g = rng.standard_normal(10)
+    lr, m = 0.3, 0.7
+    w, v = w0.copy(), np.zeros(10)
+    for k in range(1, 8):
+        w, v = O.momentum_update(w, v, g, lr, m)
+        np.testing.assert_allclose(v, lr * g * (1 - m ** k) / (1 - m), rtol=1e-13)
+        geo = sum((1 - m ** j) / (1 - m) for j in range(1, k + 1))
+        np.testing.assert_allclose(w, w0 + lr * g * geo, rtol=1e-12, atol=1e-13)
+
+
+def test_one_weight_net_two_steps_by_hand():
+    # 1-1 net: o = sigma(w x + b); delta = (t - o) o (1 - o);
+    # G_w = delta x, G_b = delta; v <- lr G + m v; w <- w + v
+    w, b, x, t, lr, m = 0.4, -0.2, 1.5, 1.0, 0.5, 0.9
+    st = O.State((1, 1), np.array([w, b]), lr=lr, momentum=m)
+    vw = vb = 0.0
+    for _ in range(2):
+        o = 1.0 / (1.0 + math.exp(-(w * x + b)))
+        d = (t - o) * o * (1 - o)
+        e = O.train_batch(st, np.array([[x]]), np.array([[t]]))
+        assert e == pytest.approx((t - o) ** 2, rel=1e-14)
+        vw, vb = lr * d * x + m * vw, lr * d + m * vb
+        w, b = w + vw, b + vb
+        np.testing.assert_allclose(st.theta, [w, b], rtol=1e-14)
+        np.testing.assert_allclose(st.V, [vw, vb], rtol=1e-14)
+
+
+def test_xor_converges():
+    # a 2-2-1 net trained with pooled updates learns XOR
+    X = np.array([[0, 0], [0, 1], [1, 0], [1, 1]], float)
+    T = np.array([[0], [1], [1], [0]], float)
+    st = O.State((2, 2, 1), synth.init_uniform((2, 2, 1), -1, 1, 2), lr=0.5, momentum=0.9)
+    for _ in range(3000):
+        e = O.train_batch(st, X, T)
+    assert e < 0.04
+    assert np.all(np.abs(O.predict(st, X) - T) < 0.2)
+
+
+def test_mean_scaling_equals_scaled_learning_rate():
+    sizes = (5, 4, 3)
+    X, T = synth.gaussian_patterns(8, 5, 3, 0.5, seed=8)
+    th = synth.init_uniform(sizes, -0.5, 0.5, 8)
+    a = O.State(sizes, th, lr=0.2, momentum=0.5, grad_scale=1.0 / 8)
+    b = O.State(sizes, th, lr=0.2 / 8, momentum=0.5)
+    for _ in range(3):
+        O.train_batch(a, X, T)
+        O.train_batch(b, X, T)
+    np.testing.assert_allclose(a.theta, b.theta, rtol=1e-12)
+
+
+def test_epoch_takes_minibatches_in_index_order():
+    sizes = (5, 4, 3)
+    X, T = synth.gaussian_patterns(10, 5, 3, 0.5, seed=9)
+    th = synth.init_uniform(sizes, -0.5, 0.5, 9)
+    a = O.State(sizes, th, 0.1, 0.9)
+    errs = O.train_epoch(a, X, T, minibatch=4)
+    assert len(errs) == 3            # 4 + 4 + ragged 2
+    b = O.State(sizes, th, 0.1, 0.9)
+    for sl in (slice(0, 4), slice(4, 8), slice(8, 10)):
+        O.train_batch(b, X[sl], T[sl])
+    np.testing.assert_array_equal(a.theta, b.theta)
+    c = O.State(sizes, th, 0.1, 0.9)
+    assert O.train_epoch(c, X, T, minibatch=10)[0] == pytest.approx(
+        O.sse(O.forward(*O.unpack(sizes, th), X)[-1], T))
+
+
+def test_pack_unpack_round_trip():
+    sizes = (3, 4, 2)
+    th = np.arange(O.connections(sizes), dtype=float)
+    Ws, bs = O.unpack(sizes, th)
+    assert Ws[0].shape == (4, 3) and bs[0].shape == (4,)
+    assert Ws[0][1, 0] == 3.0 and bs[0][0] == 12.0   # W_1 row-major, then b_1
+    np.testing.assert_array_equal(O.pack(Ws, bs), th)
+
+
+# ------------------------------------------------------------------ inputs
+def test_nettalk_patterns_structure():
+    X, T = synth.nettalk_patterns(257, seed=0)
+    assert X.shape == (257, 203) and T.shape == (257, 26)
+    blocks = X.reshape(257, 7, 29)
+    assert np.all(blocks.sum(axis=2) == 1)
+    assert np.all(T.sum(axis=1) == 3)
+    assert set(np.unique(X)) <= {0.0, 1.0}
+
+
+def test_bf16_rounding_matches_torch():
+    torch = pytest.importorskip("torch")
+    x = np.random.default_rng(0).standard_normal(10000) * 10
+    ref = torch.tensor(x, dtype=torch.float32).to(torch.bfloat16).to(torch.float64).numpy()
+    np.testing.assert_array_equal(synth.bf16_round(x), ref)
