@@ -1,0 +1,154 @@
+/*
+ * bp.h -- C ABI of libbp.so: the batch back-propagation training step of a
+ * fully connected sigmoid multi-layer perceptron on one GB300 (sm_103a).
+ *
+ * The method is the one of Witbrock & Zagha, "An Implementation of
+ * Back-Propagation Learning on GF11" (CMU-CS-89-208):
+ *   - forward pass: a_j = 1 / (1 + exp(-(sum_i w_ji a_i + b_j)))       (Section 3, fn. 4)
+ *   - error: summed squared difference E = sum (t - o)^2              (Section 3, fn. 5)
+ *   - output delta (t - o) o (1 - o); hidden delta (W^T delta) h (1 - h);
+ *     no delta for input units (Section 6.1, "Cycles backward/case")
+ *   - pooled weight change summed over every pattern of a group       (Sections 3, 4.1)
+ *   - update with learning rate and momentum, then the pooled change
+ *     is zeroed (Section 6.2.1):
+ *         V <- lr * grad_scale * G + momentum * V ;  W <- W + V ;  G <- 0
+ *     G is the pooled sum of delta * activation (minus the gradient of E/2),
+ *     V starts at zero, grad_scale is 1 (a sum, as the paper pools) unless set.
+ * The bias of a unit is its weight from the always-on "true" unit (Section 6.3)
+ * and is trained and counted like every other connection.
+ *
+ * Conventions shared by every entry point
+ *   - Layer sizes n_0 (inputs) ... n_L (outputs), 2 <= n_layers <= BP_MAX_SIZES.
+ *   - Parameter vectors ("theta", and V, G of the same shape) are flat float32
+ *     arrays in layer order: for l = 1..L, W_l as n_l rows of n_{l-1} floats
+ *     (row-major), then the n_l bias weights b_l.  Length = bp_num_params().
+ *   - Patterns are row-major: X is [batch, n_0], T and Y are [batch, n_L].
+ *     Their element type is float32 for BP_F32 nets and bfloat16 (raw uint16
+ *     bits, round-to-nearest-even) for BP_BF16 nets.  Targets are in [0, 1].
+ *   - Device pointers ("d_") are caller-owned CUDA device memory on the current
+ *     device; the library never frees them.  Host pointers ("h_") are caller-
+ *     owned host memory (pinned memory makes the copies asynchronous).
+ *   - `stream` is a cudaStream_t passed as void* (NULL = legacy default stream).
+ *     Compute entry points are asynchronous with respect to the host; the
+ *     device buffers they read must stay valid until the stream reaches them.
+ *   - A net must not be used from two host threads at once.
+ *   - Every call returns a bp_status; on failure bp_last_error() holds a
+ *     message for the calling thread.  Argument errors are detected before any
+ *     work is queued.  Errors raised by a kernel (a bounded device-side wait
+ *     that ran out, a non-finite error sum) are latched on the device and
+ *     reported by bp_check().
+ */
+#ifndef BP_H
+#define BP_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define BP_MAX_SIZES 9            /* n_0 .. n_8: at most 8 weight layers */
+
+typedef struct bp_net bp_net;     /* opaque; owns device W, b, V, G and scratch */
+
+typedef enum {
+    BP_OK = 0,
+    BP_EINVAL = 1,      /* NULL pointer, size <= 0, batch above capacity, bad hparam */
+    BP_ENOMEM = 2,      /* a device or host allocation failed */
+    BP_ECUDA = 3,       /* a CUDA runtime/driver call failed (message in bp_last_error) */
+    BP_ESHAPE = 4,      /* layer sizes or batch not supported by this net's dtype path */
+    BP_ETIMEOUT = 5,    /* a bounded device-side wait ran out; that launch did no more work */
+    BP_ENONFINITE = 6,  /* the error sum of a group came out NaN or Inf */
+    BP_ESTATE = 7       /* call order violated (e.g. bp_backward without bp_forward) */
+} bp_status;
+
+typedef enum {
+    BP_F32 = 0,   /* float32 everywhere; SIMT FFMA kernels */
+    BP_BF16 = 1   /* bfloat16 activations/deltas/weight copies on tcgen05 tensor
+                     cores with float32 accumulation; float32 master W, b, V, G */
+} bp_dtype;
+
+/* Create a net.  Weights, V and G start at zero (set them with bp_set_weights).
+ * layer_sizes: host array of n_layers ints, each >= 1.
+ * dtype: a bp_dtype.  BP_BF16 needs every n_l to be a multiple of 8.
+ * max_batch: the largest group any later call may pass (sizes device scratch).
+ * Errors: BP_EINVAL (bad argument), BP_ESHAPE (sizes unsupported by dtype),
+ * BP_ENOMEM, BP_ECUDA.  *out is set only on BP_OK. */
+bp_status bp_create(const int* layer_sizes, int n_layers, float lr, float momentum,
+                    int dtype, int max_batch, bp_net** out);
+
+/* Free every device buffer of the net.  NULL-safe.  Synchronises the device. */
+void bp_destroy(bp_net* net);
+
+/* Learning rate, momentum and the factor applied to G in the update
+ * (1 = the paper's pooled sum, 1/B = a mean).  Takes effect for work queued
+ * after the call.  Errors: BP_EINVAL if a value is not finite. */
+bp_status bp_set_hparams(bp_net* net, float lr, float momentum, float grad_scale);
+
+/* Number of float32 values in a parameter vector (W and b of every layer). */
+int64_t bp_num_params(const bp_net* net);
+
+/* Synchronous copies between host float32 arrays of bp_num_params() values and
+ * the net's weights (theta), previous weight change (V) or pending pooled
+ * change (G).  They synchronise the device first.  bp_set_weights also
+ * refreshes the bfloat16 weight copies of a BP_BF16 net. */
+bp_status bp_set_weights(bp_net* net, const float* h_theta);
+bp_status bp_get_weights(const bp_net* net, float* h_theta);
+bp_status bp_set_velocity(bp_net* net, const float* h_v);
+bp_status bp_get_velocity(const bp_net* net, float* h_v);
+bp_status bp_get_grads(const bp_net* net, float* h_g);
+
+/* Forward pass (Section 3) of `batch` patterns d_X [batch, n_0] -> d_Y
+ * [batch, n_L].  d_Y may be NULL.  The activations of every layer are kept in
+ * the net's scratch for a following bp_backward, which also reads d_X again:
+ * d_X must stay unchanged until then.  Errors: BP_EINVAL (batch < 1 or above
+ * max_batch, NULL d_X), BP_ECUDA. */
+bp_status bp_forward(bp_net* net, const void* d_X, int batch, void* d_Y, void* stream);
+
+/* Backward pass for the group of the last bp_forward: output and hidden deltas
+ * against targets d_T [batch, n_L], then G += the group's pooled change
+ * (Sections 3, 4.1).  batch must equal the last forward's.  If d_sse is not
+ * NULL, one float (the group's summed squared error) is written there.
+ * Errors: BP_ESTATE (no forward, or a different batch), BP_EINVAL, BP_ECUDA. */
+bp_status bp_backward(bp_net* net, const void* d_T, int batch, float* d_sse, void* stream);
+
+/* Apply the pending pooled change: V <- lr*grad_scale*G + momentum*V;
+ * W <- W + V; G <- 0 (Section 6.2.1). */
+bp_status bp_update(bp_net* net, void* stream);
+
+/* One whole training step on one group: forward, backward, pooled change and
+ * update, with any change already pending in G folded in.  Same buffers and
+ * errors as bp_forward + bp_backward. */
+bp_status bp_train_batch(bp_net* net, const void* d_X, const void* d_T, int batch,
+                         float* d_sse, void* stream);
+
+/* One pass over n_patterns patterns taken in index order, one update per
+ * minibatch (a ragged last minibatch is a group of its own), all queued as a
+ * single device launch.  d_sse (may be NULL) receives ceil(n_patterns /
+ * minibatch) floats, the error sum of each group.  minibatch <= max_batch.
+ * Errors: BP_EINVAL, BP_ECUDA. */
+bp_status bp_train_epoch(bp_net* net, const void* d_X, const void* d_T, int n_patterns,
+                         int minibatch, float* d_sse, void* stream);
+
+/* bp_train_epoch on HOST buffers: copies h_X and h_T to device staging owned by
+ * the net (grown on demand), runs the epoch, copies the ceil(n_patterns /
+ * minibatch) error sums back to h_sse (may be NULL) and waits for the stream.
+ * Errors as bp_train_epoch, plus BP_ENOMEM for the staging buffers and any
+ * error latched by the epoch's kernels (as bp_check). */
+bp_status bp_train_epoch_host(bp_net* net, const void* h_X, const void* h_T, int n_patterns,
+                              int minibatch, float* h_sse, void* stream);
+
+/* Wait for `stream`, then report and clear errors latched by earlier kernels:
+ * BP_ETIMEOUT if a bounded wait ran out, BP_ENONFINITE if an error sum was not
+ * finite, else BP_OK (or BP_ECUDA for an error from the CUDA runtime). */
+bp_status bp_check(bp_net* net, void* stream);
+
+/* Message describing the last failure on the calling thread ("" if none). */
+const char* bp_last_error(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* BP_H */

@@ -1,0 +1,325 @@
+"""float32 CUDA path against the float64 oracle, through the C ABI.
+
+Tolerance (fp32 SIMT path): normwise relative error
+    max|x_gpu - x_ref| / max|x_ref| <= 1e-5
+on outputs, pooled changes, error sums and weight changes, for one step from
+identical weights (elementwise relative error is ill-posed where a sigmoid
+saturates).  Inputs are seeded and synthetic (NETtalk-shaped or Gaussian).
+"""
+import numpy as np
+import pytest
+
+from oracle import bp_oracle as O
+from paper_1801_01554_gb300 import bp, synth
+
+torch = pytest.importorskip("torch")
+pytestmark = pytest.mark.gpu
+
+TOL = 1e-5
+
+
+def normwise(x, y):
+    x = np.asarray(x, dtype=np.float64)
+    y = np.asarray(y, dtype=np.float64)
+    return float(np.max(np.abs(x - y)) / max(np.max(np.abs(y)), 1e-30))
+
+
+def dev(a):
+    return torch.tensor(np.asarray(a), dtype=torch.float32, device="cuda")
+
+
+def problem(sizes, B, seed=0, lo=-0.3, hi=0.3):
+    if sizes[0] == 203 and sizes[-1] == 26:
+        X, T = synth.nettalk_patterns(B, seed=seed)
+    else:
+        X, T = synth.gaussian_patterns(B, sizes[0], sizes[-1], 0.3, seed=seed)
+        X = synth.round_to(X, "f32")
+    theta = synth.round_to(synth.init_uniform(sizes, lo, hi, seed), "f32")
+    return X, T, theta
+
+
+SHAPES = [((203, 60, 26), 1), ((203, 60, 26), 37), ((203, 60, 26), 1024),
+          ((203, 120, 26), 512), ((203, 120, 26), 1000), ((5, 3, 2), 7),
+          ((64, 33, 17, 9), 300), ((40, 300, 200, 1), 257)]
+
+
+@pytest.mark.parametrize("sizes,B", SHAPES)
+def test_forward_backward_update_match_oracle(sizes, B):
+    X, T, theta = problem(sizes, B, seed=B)
+    st = O.State(sizes, theta, lr=0.1, momentum=0.9)
+    As, Ds, G_ref, e_ref = O.step_quantities(st, X, T)
+    Xd, Td = dev(X), dev(T)
+    Yd = torch.empty((B, sizes[-1]), device="cuda")
+    sse = torch.zeros(1, device="cuda")
+    with bp.Net(sizes, 0.1, 0.9, bp.BP_F32, max_batch=B) as net:
+        net.set_weights(theta)
+        net.forward(Xd, B, Yd)
+        net.backward(Td, B, sse)
+        net.check()
+        G = net.get_grads()
+        assert normwise(Yd.cpu().numpy(), As[-1]) <= TOL
+        assert normwise(G, G_ref) <= TOL
+        assert abs(sse.item() - e_ref) <= TOL * e_ref
+        net.update()
+        net.check()
+        st.G = G_ref
+        O.apply_update(st)
+        th = net.get_weights()
+        assert normwise(th - theta, st.theta - theta) <= TOL
+        assert normwise(net.get_velocity(), st.V) <= TOL
+        assert not net.get_grads().any()          # the update zeroes G
+
+
+@pytest.mark.parametrize("sizes,B", [((203, 60, 26), 1024), ((203, 120, 26), 512),
+                                     ((203, 120, 26), 77), ((64, 33, 17, 9), 300)])
+def test_train_batch_matches_oracle(sizes, B):
+    X, T, theta = problem(sizes, B, seed=3)
+    st = O.State(sizes, theta, lr=0.05, momentum=0.9)
+    with bp.Net(sizes, 0.05, 0.9, bp.BP_F32, max_batch=B) as net:
+        net.set_weights(theta)
+        sse = torch.zeros(3, device="cuda")
+        for k in range(3):
+            net.train_batch(dev(X), dev(T), B, sse[k:k + 1])
+        net.check()
+        e_ref = [O.train_batch(st, X, T) for _ in range(3)]
+        np.testing.assert_allclose(sse.cpu().numpy(), e_ref, rtol=TOL)
+        assert normwise(net.get_weights() - theta, st.theta - theta) <= TOL
+        assert normwise(net.get_velocity(), st.V) <= TOL
+
+
+def test_pending_change_is_folded_into_train_batch():
+    sizes, B = (203, 60, 26), 200
+    X, T, theta = problem(sizes, B, seed=4)
+    X2, T2, _ = problem(sizes, B, seed=5)
+    st = O.State(sizes, theta, lr=0.1, momentum=0.5)
+    with bp.Net(sizes, 0.1, 0.5, bp.BP_F32, max_batch=B) as net:
+        net.set_weights(theta)
+        Xd = dev(X)                      # must outlive the matching bp_backward
+        net.forward(Xd, B)
+        net.backward(dev(T), B)
+        net.train_batch(dev(X2), dev(T2), B)
+        net.check()
+        O.backward_accumulate(st, X, T)
+        O.train_batch(st, X2, T2)
+        assert normwise(net.get_weights() - theta, st.theta - theta) <= TOL
+        assert not net.get_grads().any()
+
+
+def test_backward_accumulates_across_groups():
+    sizes, B = (203, 60, 26), 100
+    X, T, theta = problem(sizes, B, seed=6)
+    st = O.State(sizes, theta, lr=0.1, momentum=0.9)
+    G_ref = O.step_quantities(st, X, T)[2]
+    with bp.Net(sizes, 0.1, 0.9, bp.BP_F32, max_batch=B) as net:
+        net.set_weights(theta)
+        Xd, Td = dev(X), dev(T)
+        for _ in range(2):
+            net.forward(Xd, B)
+            net.backward(Td, B)
+        net.check()
+        assert normwise(net.get_grads(), 2 * G_ref) <= TOL
+
+
+@pytest.mark.parametrize("n,mb", [(4096, 512), (1000, 300), (777, 1)])
+def test_train_epoch_matches_oracle(n, mb):
+    sizes = (203, 120, 26)
+    X, T, theta = problem(sizes, n, seed=7)
+    st = O.State(sizes, theta, lr=0.05, momentum=0.9)
+    e_ref = O.train_epoch(st, X, T, mb)
+    with bp.Net(sizes, 0.05, 0.9, bp.BP_F32, max_batch=mb) as net:
+        net.set_weights(theta)
+        sse = torch.zeros(len(e_ref), device="cuda")
+        net.train_epoch(dev(X), dev(T), n, mb, sse)
+        net.check()
+        np.testing.assert_allclose(sse.cpu().numpy(), e_ref, rtol=1e-4, atol=1e-6)
+        assert normwise(net.get_weights() - theta, st.theta - theta) <= 1e-4
+
+
+@pytest.mark.parametrize("B", synth.SWEEP_BATCHES)
+def test_batch_sweep_step_matches_oracle(B):
+    sizes = (203, 120, 26)
+    X, T, theta = problem(sizes, B, seed=11)
+    V0 = synth.round_to(np.random.default_rng(2).uniform(-1e-3, 1e-3, theta.size), "f32")
+    st = O.State(sizes, theta, lr=0.05, momentum=0.9, V=V0.copy())
+    e_ref = O.train_batch(st, X, T)
+    with bp.Net(sizes, 0.05, 0.9, bp.BP_F32, max_batch=B) as net:
+        net.set_weights(theta)
+        net.set_velocity(V0)
+        sse = torch.zeros(1, device="cuda")
+        net.train_batch(dev(X), dev(T), B, sse)
+        net.check()
+        assert abs(sse.item() - e_ref) <= TOL * e_ref
+        assert normwise(net.get_weights() - theta, st.theta - theta) <= TOL
+        assert normwise(net.get_velocity(), st.V) <= TOL
+
+
+def test_mean_scaling():
+    sizes, B = (203, 60, 26), 256
+    X, T, theta = problem(sizes, B, seed=12)
+    st = O.State(sizes, theta, lr=0.1, momentum=0.9, grad_scale=1.0 / B)
+    with bp.Net(sizes, 0.1, 0.9, bp.BP_F32, max_batch=B, grad_scale=1.0 / B) as net:
+        net.set_weights(theta)
+        for _ in range(2):
+            net.train_batch(dev(X), dev(T), B)
+            O.train_batch(st, X, T)
+        net.check()
+        assert normwise(net.get_weights() - theta, st.theta - theta) <= TOL
+
+
+def test_zero_learning_rate_keeps_weights_bitwise():
+    sizes, B = (203, 60, 26), 64
+    X, T, theta = problem(sizes, B, seed=13)
+    with bp.Net(sizes, 0.0, 0.9, bp.BP_F32, max_batch=B) as net:
+        net.set_weights(theta)
+        net.train_epoch(dev(X), dev(T), B, 16)
+        net.check()
+        np.testing.assert_array_equal(net.get_weights(), theta.astype(np.float32))
+
+
+def test_runs_are_bitwise_reproducible():
+    sizes, n, mb = (203, 120, 26), 2048, 512
+    X, T, theta = problem(sizes, n, seed=14)
+    out = []
+    for _ in range(2):
+        with bp.Net(sizes, 0.05, 0.9, bp.BP_F32, max_batch=mb) as net:
+            net.set_weights(theta)
+            net.train_epoch(dev(X), dev(T), n, mb)
+            net.check()
+            out.append(net.get_weights())
+    np.testing.assert_array_equal(out[0], out[1])
+
+
+def test_pooled_change_is_order_independent_on_gpu():
+    # Section 4.1: patterns may be presented in any order
+    sizes, B = (203, 120, 26), 512
+    X, T, theta = problem(sizes, B, seed=15)
+    perm = np.random.default_rng(0).permutation(B)
+    Gs = []
+    for Xp, Tp in ((X, T), (X[perm], T[perm])):
+        with bp.Net(sizes, 0.05, 0.9, bp.BP_F32, max_batch=B) as net:
+            net.set_weights(theta)
+            Xd = dev(Xp)
+            net.forward(Xd, B)
+            net.backward(dev(Tp), B)
+            Gs.append(net.get_grads())
+    assert normwise(Gs[1], Gs[0]) <= TOL
+
+
+def test_checkpoint_resume_is_exact():
+    sizes, n, mb = (203, 60, 26), 1024, 256
+    X, T, theta = problem(sizes, n, seed=16)
+    Xd, Td = dev(X), dev(T)
+    with bp.Net(sizes, 0.1, 0.9, bp.BP_F32, max_batch=mb) as a:
+        a.set_weights(theta)
+        a.train_epoch(Xd, Td, n, mb)
+        w, v = a.get_weights(), a.get_velocity()
+        a.train_epoch(Xd, Td, n, mb)
+        ref = a.get_weights()
+    with bp.Net(sizes, 0.1, 0.9, bp.BP_F32, max_batch=mb) as b:
+        b.set_weights(w)
+        b.set_velocity(v)
+        b.train_epoch(Xd, Td, n, mb)
+        np.testing.assert_array_equal(b.get_weights(), ref)
+
+
+def test_host_buffer_epoch_equals_device_epoch():
+    sizes, n, mb = (203, 120, 26), 3000, 512
+    X, T, theta = problem(sizes, n, seed=17)
+    Xh = torch.tensor(X, dtype=torch.float32).pin_memory()
+    Th = torch.tensor(T, dtype=torch.float32).pin_memory()
+    sse_h = np.zeros(6, dtype=np.float32)
+    with bp.Net(sizes, 0.05, 0.9, bp.BP_F32, max_batch=mb) as a:
+        a.set_weights(theta)
+        a.train_epoch_host(Xh, Th, n, mb, sse_h)
+        wa = a.get_weights()
+    with bp.Net(sizes, 0.05, 0.9, bp.BP_F32, max_batch=mb) as b:
+        b.set_weights(theta)
+        sse_d = torch.zeros(6, device="cuda")
+        b.train_epoch(dev(X), dev(T), n, mb, sse_d)
+        np.testing.assert_array_equal(b.get_weights(), wa)
+        np.testing.assert_array_equal(sse_d.cpu().numpy(), sse_h)
+
+
+def test_argument_and_state_errors():
+    sizes = (203, 60, 26)
+    with bp.Net(sizes, 0.1, 0.9, bp.BP_F32, max_batch=16) as net:
+        X = torch.zeros((32, 203), device="cuda")
+        T = torch.zeros((32, 26), device="cuda")
+        with pytest.raises(bp.BPError) as e:
+            net.forward(X, 32)
+        assert e.value.status == bp.BP_EINVAL
+        with pytest.raises(bp.BPError) as e:
+            net.backward(T, 8)
+        assert e.value.status == bp.BP_ESTATE
+        net.forward(X, 8)
+        with pytest.raises(bp.BPError) as e:
+            net.backward(T, 4)
+        assert e.value.status == bp.BP_ESTATE
+        with pytest.raises(bp.BPError) as e:
+            net.train_epoch(X, T, 0, 8)
+        assert e.value.status == bp.BP_EINVAL
+        with pytest.raises(bp.BPError) as e:
+            net.set_hparams(float("nan"), 0.9)
+        assert e.value.status == bp.BP_EINVAL
+        net.check()
+
+
+def test_nonfinite_error_sum_is_reported():
+    sizes, B = (4, 3, 2), 8
+    X = np.full((B, 4), np.nan)
+    T = np.zeros((B, 2))
+    with bp.Net(sizes, 0.1, 0.9, bp.BP_F32, max_batch=B) as net:
+        net.set_weights(np.full(bp.connections(sizes), 0.1))
+        net.train_batch(dev(X), dev(T), B)
+        with pytest.raises(bp.BPError) as e:
+            net.check()
+        assert e.value.status == bp.BP_ENONFINITE
+        net.check()    # the latch is cleared
+
+
+def test_nettalk60_workload_full():
+    """203-60-26, 1,024 patterns, full-batch updates, lr 0.1, momentum 0.9, 10 epochs."""
+    sizes, X, T, theta = synth.make_workload("nettalk60")
+    w = synth.WORKLOADS["nettalk60"]
+    st = O.State(sizes, theta, lr=w["lr"], momentum=w["momentum"])
+    n = len(X)
+    with bp.Net(sizes, w["lr"], w["momentum"], bp.BP_F32, max_batch=n) as net:
+        net.set_weights(theta)
+        sse = torch.zeros(w["epochs"], device="cuda")
+        Xd, Td = dev(X), dev(T)
+        for ep in range(w["epochs"]):
+            net.train_epoch(Xd, Td, n, w["minibatch"], sse[ep:ep + 1])
+            e_ref = O.train_epoch(st, X, T, w["minibatch"])[0]
+            # each epoch's error sum is compared on the trajectory so far
+            assert abs(sse[ep].item() - e_ref) <= 1e-4 * e_ref, ep
+        net.check()
+        assert normwise(net.get_weights() - theta, st.theta - theta) <= 1e-4
+
+
+@pytest.mark.slow
+def test_nettalk120_workload_full():
+    """203-120-26, 65,536 patterns, minibatch 512, lr 0.05, momentum 0.9, 5 epochs, launched
+    as the benchmark launches it (one persistent launch per epoch)."""
+    sizes, X, T, theta = synth.make_workload("nettalk120")
+    w = synth.WORKLOADS["nettalk120"]
+    n, mb = len(X), w["minibatch"]
+    st = O.State(sizes, theta, lr=w["lr"], momentum=w["momentum"])
+    Xd, Td = dev(X), dev(T)
+    steps = n // mb
+    with bp.Net(sizes, w["lr"], w["momentum"], bp.BP_F32, max_batch=mb) as net:
+        net.set_weights(theta)
+        sse = torch.zeros(w["epochs"] * steps, device="cuda")
+        for ep in range(w["epochs"]):
+            net.train_epoch(Xd, Td, n, mb, sse[ep * steps:(ep + 1) * steps])
+        net.check()
+        e_gpu = sse.cpu().numpy()
+        th = net.get_weights()
+    e_ref = []
+    for ep in range(w["epochs"]):
+        e_ref += O.train_epoch(st, X, T, mb)
+    e_ref = np.array(e_ref)
+    rel = np.abs(e_gpu - e_ref) / e_ref
+    print("max rel SSE error over", len(e_ref), "updates:", rel.max(),
+          "weight-change error:", normwise(th - theta, st.theta - theta))
+    assert rel.max() <= TOL
+    assert normwise(th - theta, st.theta - theta) <= TOL
