@@ -71,7 +71,8 @@ typedef enum {
 
 /* Create a net.  Weights, V and G start at zero (set them with bp_set_weights).
  * layer_sizes: host array of n_layers ints, each >= 1.
- * dtype: a bp_dtype.  BP_BF16 needs every n_l to be a multiple of 8.
+ * dtype: a bp_dtype.  BP_BF16 needs every n_l to be a multiple of 8 (16-byte
+ * rows for the tensor-memory copies); any batch size works.
  * max_batch: the largest group any later call may pass (sizes device scratch).
  * Errors: BP_EINVAL (bad argument), BP_ESHAPE (sizes unsupported by dtype),
  * BP_ENOMEM, BP_ECUDA.  *out is set only on BP_OK. */
@@ -124,8 +125,9 @@ bp_status bp_train_batch(bp_net* net, const void* d_X, const void* d_T, int batc
                          float* d_sse, void* stream);
 
 /* One pass over n_patterns patterns taken in index order, one update per
- * minibatch (a ragged last minibatch is a group of its own), all queued as a
- * single device launch.  d_sse (may be NULL) receives ceil(n_patterns /
+ * minibatch (a ragged last minibatch is a group of its own).  A BP_F32 net runs
+ * the whole pass as one persistent device launch; a BP_BF16 net queues one
+ * chain of tensor-core kernels per minibatch.  d_sse (may be NULL) receives ceil(n_patterns /
  * minibatch) floats, the error sum of each group.  minibatch <= max_batch.
  * Errors: BP_EINVAL, BP_ECUDA. */
 bp_status bp_train_epoch(bp_net* net, const void* d_X, const void* d_T, int n_patterns,
