@@ -146,6 +146,37 @@ bp_status bp_train_epoch_host(bp_net* net, const void* h_X, const void* h_T, int
  * finite, else BP_OK (or BP_ECUDA for an error from the CUDA runtime). */
 bp_status bp_check(bp_net* net, void* stream);
 
+/* bp_train_epoch for callers that cannot allocate device memory.  The paper
+ * has no counterpart to this entry point; it exists for callers such as code
+ * running inside a host framework that owns the device allocator, processes
+ * whose device memory budget was handed out up front, or plug-ins that may only
+ * touch the buffers given to them.  It creates no bp_net and calls no
+ * cudaMalloc, cudaFree or other allocating routine.
+ *   Float32 nets only.  The caller passes every input and output:
+ *     d_theta, d_V  float32 [bp_num_params] weights and previous weight change,
+ *                   read and updated in place (start d_V at zero);
+ *     d_X, d_T      float32 patterns [n_patterns, n_0] and targets [n_patterns, n_L];
+ *     d_sse         NULL or ceil(n_patterns / minibatch) floats: error sums;
+ *     d_status      NULL or one int: 0 when the launch finished cleanly, else the
+ *                   latched error bits (1 = a bounded wait ran out, 2 = a
+ *                   non-finite error sum).
+ *   Scratch (activations, deltas, barrier, error word) lives in one static
+ *   device array of 8 MiB, which every GPU that loads the library holds until the
+ *   process exits.  Sizes whose scratch, 4 * (16 + SMs + 2 * minibatch *
+ *   sum_l roundup4(n_l)) bytes, exceeds 8 MiB are rejected with BP_EINVAL (for
+ *   203-120-26 a minibatch of up to about 7,000 patterns fits).
+ *   The first call on a device looks up the array's device address and sets
+ *   kernel attributes; make that first call before any stream capture.  All
+ *   calls on a device share the array and find the previous call's contents:
+ *   the call clears what must start at zero, and calls that overlap on the GPU
+ *   (different streams, or several host threads) race on it.
+ *   Asynchronous with respect to the host like bp_train_epoch.  Errors:
+ *   BP_EINVAL, BP_ESHAPE, BP_ECUDA. */
+bp_status bp_train_epoch_noalloc(const int* layer_sizes, int n_layers, float lr, float momentum,
+                                 float grad_scale, float* d_theta, float* d_V, const float* d_X,
+                                 const float* d_T, int n_patterns, int minibatch, float* d_sse,
+                                 int* d_status, void* stream);
+
 /* Message describing the last failure on the calling thread ("" if none). */
 const char* bp_last_error(void);
 

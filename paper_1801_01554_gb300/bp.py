@@ -43,6 +43,8 @@ SIGNATURES = {
     "bp_train_epoch": (_I, [_VP, _VP, _VP, _I, _I, _VP, _VP]),
     "bp_train_epoch_host": (_I, [_VP, _VP, _VP, _I, _I, _FP, _VP]),
     "bp_check": (_I, [_VP, _VP]),
+    "bp_train_epoch_noalloc": (_I, [ctypes.POINTER(_I), _I, _F, _F, _F, _VP, _VP, _VP, _VP, _I, _I,
+                                    _VP, _VP, _VP]),
     "bp_last_error": (ctypes.c_char_p, []),
 }
 
@@ -209,6 +211,18 @@ def bp_train_epoch_host(h, X, T, n_patterns, minibatch, sse=None, stream=None):
 
 def bp_check(h, stream=None):
     _check(load().bp_check(h, _stream(stream)))
+
+
+def bp_train_epoch_noalloc(sizes, lr, momentum, grad_scale, theta, V, X, T, n_patterns, minibatch,
+                           sse=None, status=None, stream=None):
+    """Training epoch that allocates nothing: every buffer is the caller's
+    (float32 CUDA tensors theta and V are updated in place)."""
+    sizes = [int(s) for s in sizes]
+    arr = (ctypes.c_int * len(sizes))(*sizes)
+    _check(load().bp_train_epoch_noalloc(arr, len(sizes), float(lr), float(momentum),
+                                         float(grad_scale), _dptr(theta), _dptr(V), _dptr(X),
+                                         _dptr(T), int(n_patterns), int(minibatch), _dptr(sse),
+                                         _dptr(status), _stream(stream)))
 
 
 def bp_last_error() -> str:

@@ -436,3 +436,8 @@ bp_status bp_train_epoch_host(bp_net* net, const void* h_X, const void* h_T, int
 }
 
 }  // extern "C"
+
+namespace bp {
+// Lets other translation units report a message through bp_last_error().
+void set_error_message(const char* msg) { g_err = msg; }
+}  // namespace bp

@@ -66,4 +66,7 @@ cudaError_t f32_train(const F32View& v, const float* X, const float* T, int n_pa
                       int minibatch, int n_steps, float* sse_out, bool fold_g,
                       const F32Plan& plan, cudaStream_t s);
 
+// Message returned by bp_last_error() on the calling thread (bp_api.cu).
+void set_error_message(const char* msg);
+
 }  // namespace bp

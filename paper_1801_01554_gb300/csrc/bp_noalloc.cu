@@ -1,0 +1,165 @@
+// bp_train_epoch_noalloc: the float32 training launch for callers that cannot
+// allocate device memory.
+//
+// Some callers cannot call cudaMalloc at all: code running inside a captured
+// region of a host framework that owns the allocator, memory-budgeted
+// processes whose device memory was handed out up front, or plug-ins that may
+// only touch buffers given to them.  This entry point takes every input and
+// output from the caller and keeps its scratch (activations, deltas, per-CTA
+// error sums, the grid barrier and the error word) in one file-scope device
+// array of fixed size instead of allocating it.
+#include <cuda_runtime.h>
+
+#include <cstdio>
+#include <mutex>
+
+#include "bp.h"
+#include "bp_internal.h"
+
+namespace bp {
+namespace {
+
+// 8 MiB of scratch.  Every GPU that loads the library holds this array until
+// the process exits; every call on a device shares it.
+constexpr size_t kNoallocScratchBytes = 8u << 20;
+constexpr size_t kNoallocScratchFloats = kNoallocScratchBytes / sizeof(float);
+
+static __device__ __align__(256) float g_noalloc_scratch[kNoallocScratchFloats];
+
+constexpr int kMaxDevices = 64;
+std::mutex g_noalloc_mu;
+float* g_scratch_addr[kMaxDevices];   // device address of the array, per device
+int g_scratch_sms[kMaxDevices];
+
+// Once per device, with that device current: the array's device address (the
+// host-side name is only a stand-in) and the kernels' shared-memory limits.
+bp_status noalloc_setup(int dev, float** addr, int* sms) {
+    std::lock_guard<std::mutex> lk(g_noalloc_mu);
+    if (g_scratch_addr[dev] == nullptr) {
+        float* p = nullptr;
+        cudaError_t e = cudaGetSymbolAddress((void**)&p, g_noalloc_scratch);
+        if (e != cudaSuccess || p == nullptr) {
+            set_error_message("bp_train_epoch_noalloc: cudaGetSymbolAddress of the static scratch failed");
+            return BP_ECUDA;
+        }
+        int n = 0;
+        e = cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev);
+        if (e == cudaSuccess) e = f32_setup(dev);
+        if (e != cudaSuccess) {
+            set_error_message("bp_train_epoch_noalloc: device set-up failed");
+            return BP_ECUDA;
+        }
+        g_scratch_sms[dev] = n;
+        g_scratch_addr[dev] = p;
+    }
+    *addr = g_scratch_addr[dev];
+    *sms = g_scratch_sms[dev];
+    return BP_OK;
+}
+
+}  // namespace
+}  // namespace bp
+
+using namespace bp;
+
+extern "C" bp_status bp_train_epoch_noalloc(const int* layer_sizes, int n_layers, float lr,
+                                            float momentum, float grad_scale, float* d_theta,
+                                            float* d_V, const float* d_X, const float* d_T,
+                                            int n_patterns, int minibatch, float* d_sse,
+                                            int* d_status, void* stream) {
+    char msg[256];
+    if (layer_sizes == nullptr || d_theta == nullptr || d_V == nullptr || d_X == nullptr ||
+        d_T == nullptr) {
+        set_error_message("bp_train_epoch_noalloc: NULL argument");
+        return BP_EINVAL;
+    }
+    if (n_layers < 2 || n_layers > BP_MAX_SIZES) {
+        set_error_message("bp_train_epoch_noalloc: n_layers out of range");
+        return BP_EINVAL;
+    }
+    for (int l = 0; l < n_layers; ++l)
+        if (layer_sizes[l] < 1) {
+            set_error_message("bp_train_epoch_noalloc: layer sizes must be >= 1");
+            return BP_EINVAL;
+        }
+    if (n_patterns < 1 || minibatch < 1) {
+        set_error_message("bp_train_epoch_noalloc: n_patterns and minibatch must be >= 1");
+        return BP_EINVAL;
+    }
+    const int L = n_layers - 1;
+    if (f32_max_pg(layer_sizes, L) < 1) {
+        set_error_message("bp_train_epoch_noalloc: one pattern's activations do not fit in shared memory");
+        return BP_ESHAPE;
+    }
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) {
+        set_error_message("bp_train_epoch_noalloc: no usable current device");
+        return BP_ECUDA;
+    }
+    float* base = nullptr;
+    int sms = 0;
+    bp_status st = noalloc_setup(dev, &base, &sms);
+    if (st != BP_OK) return st;
+
+    // scratch layout (floats, each part 16-byte aligned):
+    // [error word, pad][barrier x2, pad][per-CTA error sums][A rows][D rows]
+    F32View v{};
+    v.L = L;
+    v.cap = minibatch;
+    long long pos = 0, soff = 0;
+    int tiles = 0;
+    for (int l = 0; l <= L; ++l) v.n[l] = layer_sizes[l];
+    v.tile0[0] = v.tile0[1] = 0;
+    for (int l = 1; l <= L; ++l) {
+        v.woff[l] = pos;
+        pos += (long long)layer_sizes[l] * layer_sizes[l - 1];
+        v.boff[l] = pos;
+        pos += layer_sizes[l];
+        v.soff[l] = soff;
+        soff += (long long)minibatch * ((layer_sizes[l] + 3) & ~3);
+        const int rows = (layer_sizes[l] + 7) / 8, cols = (layer_sizes[l - 1] + 1 + 31) / 32;
+        v.tcols[l] = cols;
+        v.tile0[l] = tiles;
+        tiles += rows * cols;
+        v.tile0[l + 1] = tiles;
+    }
+    const long long head = 4 + 4 + (((long long)sms + 3) & ~3LL);
+    const long long need = head + 2 * soff;
+    if (need > (long long)kNoallocScratchFloats) {
+        snprintf(msg, sizeof msg,
+                 "bp_train_epoch_noalloc: these sizes and minibatch %d need %lld bytes of scratch; "
+                 "the static scratch holds %zu bytes (use a smaller minibatch)",
+                 minibatch, need * 4, kNoallocScratchBytes);
+        set_error_message(msg);
+        return BP_EINVAL;
+    }
+    v.flags = reinterpret_cast<int*>(base);
+    v.bar = reinterpret_cast<unsigned*>(base + 4);
+    v.sse_part = base + 8;
+    v.A = base + head;
+    v.D = base + head + soff;
+    v.theta = d_theta;
+    v.V = d_V;
+    v.G = nullptr;   // nothing pending: the launch never reads G
+    v.lr = lr;
+    v.momentum = momentum;
+    v.grad_scale = grad_scale;
+
+    cudaStream_t s = (cudaStream_t)stream;
+    // the array keeps the last call's contents: the error word and the barrier
+    // must start at zero
+    cudaError_t e = cudaMemsetAsync(base, 0, 8 * sizeof(float), s);
+    if (e == cudaSuccess) {
+        const F32Plan plan = f32_plan(v, minibatch, sms);
+        const int n_steps = (int)(((long long)n_patterns + minibatch - 1) / minibatch);
+        e = f32_train(v, d_X, d_T, n_patterns, minibatch, n_steps, d_sse, false, plan, s);
+    }
+    if (e == cudaSuccess && d_status != nullptr)
+        e = cudaMemcpyAsync(d_status, base, sizeof(int), cudaMemcpyDeviceToDevice, s);
+    if (e != cudaSuccess) {
+        snprintf(msg, sizeof msg, "bp_train_epoch_noalloc: %s", cudaGetErrorString(e));
+        set_error_message(msg);
+        return BP_ECUDA;
+    }
+    return BP_OK;
+}
