@@ -149,14 +149,15 @@ def allreduce_max(x, world, device):
 
 
 # ------------------------------------------------------------------ oracle timing
-def _oracle_child(patterns_cap, budget_s, steps=1, warmup=0, min_s=0.0, max_epochs=1):
+def _oracle_child(patterns_cap, budget_s, steps=1, warmup=0, min_s=0.0, max_epochs=1,
+                  workload=WORKLOAD):
     """Runs in a fresh interpreter with one BLAS thread: times the oracle on the
     leading `patterns_cap` patterns of the workload (one update per minibatch),
     `warmup` untimed then `steps` timed times, each bounded by `budget_s`."""
     from oracle import bp_oracle as O
     from paper_1801_01554_gb300 import synth
-    w = synth.WORKLOADS[WORKLOAD]
-    sizes, X, T, theta = synth.make_workload(WORKLOAD, patterns=patterns_cap)
+    w = synth.WORKLOADS[workload]
+    sizes, X, T, theta = synth.make_workload(workload, patterns=patterns_cap)
     st = O.State(sizes, theta, lr=w["lr"], momentum=w["momentum"])
     mb = w["minibatch"]
     out = []
@@ -177,13 +178,14 @@ def _oracle_child(patterns_cap, budget_s, steps=1, warmup=0, min_s=0.0, max_epoc
     return out
 
 
-def time_oracle(patterns_cap, budget_s, steps=1, warmup=0, min_s=0.0, max_epochs=1):
+def time_oracle(patterns_cap, budget_s, steps=1, warmup=0, min_s=0.0, max_epochs=1,
+                workload=WORKLOAD):
     env = dict(os.environ)
     for k in ("OMP_NUM_THREADS", "OPENBLAS_NUM_THREADS", "MKL_NUM_THREADS"):
         env[k] = "1"
     code = ("import json,sys; sys.path.insert(0, %r); import bench; "
-            "print(json.dumps(bench._oracle_child(%d, %f, %d, %d, %f, %d)))"
-            % (ROOT, patterns_cap, budget_s, steps, warmup, min_s, max_epochs))
+            "print(json.dumps(bench._oracle_child(%d, %f, %d, %d, %f, %d, %r)))"
+            % (ROOT, patterns_cap, budget_s, steps, warmup, min_s, max_epochs, workload))
     r = subprocess.run([sys.executable, "-c", code], env=env, capture_output=True, text=True,
                        cwd=ROOT, timeout=1800)
     if r.returncode != 0:
@@ -248,8 +250,8 @@ def run_ours(args, world, rank, local):
         raise SystemExit("bench.py needs a CUDA GPU")
     torch.cuda.set_device(local)
     device = torch.device("cuda", local)
-    w = synth.WORKLOADS[WORKLOAD]
-    sizes, X, T, theta = synth.make_workload(WORKLOAD)
+    w = synth.WORKLOADS[args.workload]
+    sizes, X, T, theta = synth.make_workload(args.workload)
     n, mb = len(X), w["minibatch"]
     updates = (n + mb - 1) // mb
     W = connections(sizes)
@@ -258,7 +260,8 @@ def run_ours(args, world, rank, local):
     # runs in its own interpreter), on rank 0 only, single-GPU runs only.
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        r = time_oracle(n, 60.0, min_s=args.cpu_seconds, max_epochs=w["epochs"])[0]
+        r = time_oracle(n, 60.0, min_s=args.cpu_seconds, max_epochs=w["epochs"],
+                        workload=args.workload)[0]
         cpu = {"value": W * r["patterns"] / r["seconds"], "unit": UNIT, "cores": 1,
                "kind": "oracle",
                "sample": f"{r['patterns']} patterns ({r['patterns'] / n:.2f} epochs of the "
@@ -354,6 +357,72 @@ def run_ours(args, world, rank, local):
     return 0
 
 
+def run_wide(args, world, rank, local):
+    """BF16 tensor-core workloads: one step = one training update on the full batch."""
+    import torch
+    from paper_1801_01554_gb300 import bp, synth
+
+    torch.cuda.set_device(local)
+    device = torch.device("cuda", local)
+    name = args.workload
+    w = synth.WORKLOADS[name]
+    sizes, X, T, theta = synth.make_workload(name)
+    B = w["minibatch"]
+    W = connections(sizes)
+    Xd = torch.tensor(X, dtype=torch.float32, device=device).to(torch.bfloat16)
+    Td = torch.tensor(T, dtype=torch.float32, device=device).to(torch.bfloat16)
+    del X, T
+    sse = torch.zeros(1, dtype=torch.float32, device=device)
+    stream = torch.cuda.current_stream(device)
+    net = bp.Net(sizes, w["lr"], w["momentum"], bp.BP_BF16, max_batch=B)
+    net.set_weights(theta)
+    for _ in range(args.warmup):
+        net.train_batch(Xd, Td, B, sse, stream)
+    net.check(stream)
+    starts = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+    ends = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+    clocks = ClockSampler(local)
+    barrier(world)
+    torch.cuda.synchronize(device)
+    clocks.start()
+    time.sleep(0.3)
+    for k in range(args.steps):
+        starts[k].record(stream)
+        net.train_batch(Xd, Td, B, sse, stream)
+        ends[k].record(stream)
+    torch.cuda.synchronize(device)
+    clk = clocks.stop()
+    net.check(stream)
+    dev_s = sum(s_.elapsed_time(e_) for s_, e_ in zip(starts, ends)) / 1e3
+    dev_s_max = allreduce_max(dev_s, world, device)
+    value = W * B * args.steps * world / dev_s_max
+    flops = algorithmic_flops_per_pattern(sizes) * B
+    achieved = flops / (dev_s / args.steps) / 1e12
+    peaks = measured_peaks()
+    peak = float(peaks.get("bf16_tflops_sustained", 1700.0))
+    net.close()
+    line = {
+        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": 1e3 * dev_s_max / args.steps,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
+        "data": "synthetic",
+        "config": {"workload": f"{'-'.join(map(str, sizes))} sigmoid MLP, bf16 activations and "
+                               f"weight copies, fp32 accumulate and master weights, batch {B}, "
+                               f"lr {w['lr']}, momentum {w['momentum']}; one step = one update",
+                   "global_batch": B, "parallelism": "single GPU",
+                   "l2": "activations of one step exceed the 129 MB L2"},
+        "roofline": {"bound": "tensor", "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
+                     "frac": achieved / peak, "traffic": None,
+                     "kernel": "whole training step (k_gemm forward, hidden-delta and pooled-change "
+                               "GEMMs, transposes, update); flops = (6W - 2W_i) per pattern",
+                     "peak_basis": "measured bf16 cuBLAS, sustained"},
+        "clocks": clk,
+    }
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    return 0
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -362,12 +431,17 @@ def main():
     ap.add_argument("--impl", choices=("ours", "reference"), default="ours")
     ap.add_argument("--cpu-seconds", type=float, default=10.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--workload", default=WORKLOAD,
+                    choices=("nettalk60", "nettalk120", "wide3", "wide4096"),
+                    help="workload to time (default: the 203-120-26 NETtalk-shaped net)")
     args = ap.parse_args()
     if args.warmup < 3 and args.impl == "ours":
         args.warmup = 3
     world, rank, local = dist_setup()
     if args.impl == "reference":
         rc = run_reference(args, world, rank)
+    elif args.workload in ("wide3", "wide4096"):
+        rc = run_wide(args, world, rank, local)
     else:
         rc = run_ours(args, world, rank, local)
     if world > 1:

@@ -416,12 +416,17 @@ __device__ void weight_phase(const F32View& v, const float* __restrict__ X, int 
     }
 }
 
+// Error sum of the group by the first warp of CTA 0: lane-strided partial sums
+// then a fixed butterfly (the same order on every run).
 __device__ void reduce_sse(const F32View& v, int nparts, float* sse_out) {
-    if (blockIdx.x == 0 && threadIdx.x == 0) {
+    if (blockIdx.x == 0 && threadIdx.x < 32) {
         float s = 0.f;
-        for (int c = 0; c < nparts; ++c) s += __ldcg(v.sse_part + c);
-        if (sse_out != nullptr) *sse_out = s;
-        if (!isfinite(s)) atomicOr(v.flags, kFlagNonfinite);
+        for (int c = threadIdx.x; c < nparts; c += 32) s += __ldcg(v.sse_part + c);
+        s = warp_sum(s);
+        if (threadIdx.x == 0) {
+            if (sse_out != nullptr) *sse_out = s;
+            if (!isfinite(s)) atomicOr(v.flags, kFlagNonfinite);
+        }
     }
 }
 

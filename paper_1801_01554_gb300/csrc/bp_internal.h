@@ -69,4 +69,54 @@ cudaError_t f32_train(const F32View& v, const float* X, const float* T, int n_pa
 // Message returned by bp_last_error() on the calling thread (bp_api.cu).
 void set_error_message(const char* msg);
 
+// --- float32 path on thread-block clusters (bp_f32_cluster.cu) -------------
+constexpr size_t kClSmemLimit = 227 * 1024 - 1024;   // dynamic shared memory per CTA
+constexpr int kClMaxCopies = 19;                     // clusters (net copies) at most
+
+// Shared-memory carve of a CTA (offsets in floats), computed on the host.
+struct ClCarve {
+    int L, C, Pc, R;
+    int slice, stg, red, total;
+    int n[BP_MAX_SIZES], ucap[BP_MAX_SIZES], nup[BP_MAX_SIZES], pf[BP_MAX_SIZES];
+    int rp[BP_MAX_SIZES], blk[BP_MAX_SIZES];
+    int wt[BP_MAX_SIZES], wsz[BP_MAX_SIZES], soff[BP_MAX_SIZES];
+    int full[BP_MAX_SIZES], dn[BP_MAX_SIZES], S[BP_MAX_SIZES], joff[BP_MAX_SIZES];
+    int sidx[BP_MAX_SIZES], ks[BP_MAX_SIZES];
+    int tin;
+};
+
+// Arguments of the cluster training kernel.
+struct ClArgs {
+    int L;
+    int n[BP_MAX_SIZES];
+    long long woff[BP_MAX_SIZES];
+    long long boff[BP_MAX_SIZES];
+    long long P;          // parameters
+    ClCarve cv;           // set from the plan at launch
+    float* theta;
+    float* V;
+    float* G;             // pending pooled change (read only when folded in)
+    float* gpart;         // [2][clusters][C][slice]: each CTA's pooled change
+    float* sse_part;      // [2][CTAs]
+    unsigned* bar;
+    int* flags;
+    float lr, momentum, grad_scale;
+};
+
+struct ClPlan {
+    bool ok;
+    int C;        // CTAs per cluster
+    int NC;       // clusters = copies of the net
+    int Pc;       // patterns per chunk
+    int R;        // copies staged per round
+    size_t smem;
+};
+
+cudaError_t cl_setup(int device);
+size_t cl_slice_floats(const int* n, int L, int C);   // floats of one CTA's slice
+ClPlan cl_plan(const int* n, int L, int batch, int num_sms);
+cudaError_t f32_train_cluster(const ClArgs& a, const float* X, const float* T, int n_patterns,
+                              int minibatch, int n_steps, float* sse_out, bool fold_g,
+                              const ClPlan& plan, cudaStream_t s);
+
 }  // namespace bp
