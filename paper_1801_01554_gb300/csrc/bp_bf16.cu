@@ -213,11 +213,46 @@ __device__ __forceinline__ void reduce_scatter32(float (&v)[32], int lane) {
 __device__ __forceinline__ void epi_bar() { asm volatile("bar.sync 1, 128;" ::: "memory"); }
 
 // ------------------------------------------------------------ epilogue
-// One 32-column chunk of one row (this thread's row m) of the tile.
+__device__ __forceinline__ void tma_store_2d(const CUtensorMap* map, const void* smem_src, int c0,
+                                             int c1) {
+    asm volatile(
+        "cp.async.bulk.tensor.2d.global.shared::cta.bulk_group [%0, {%1, %2}], [%3];" ::"l"(
+            (unsigned long long)map),
+        "r"(c0), "r"(c1), "r"(smem_u32(smem_src))
+        : "memory");
+}
+
+// 32 consecutive bf16 of one row as floats (16-byte loads when the row segment is whole).
+__device__ __forceinline__ void load_row32(float (&a)[32], const bf16* p, bool whole, int valid) {
+    if (whole) {
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {
+            const uint4 u = __ldg(reinterpret_cast<const uint4*>(p) + k);
+            const __nv_bfloat162* h = reinterpret_cast<const __nv_bfloat162*>(&u);
+#pragma unroll
+            for (int q = 0; q < 4; ++q) {
+                const float2 f = __bfloat1622float2(h[q]);
+                a[k * 8 + 2 * q] = f.x;
+                a[k * 8 + 2 * q + 1] = f.y;
+            }
+        }
+    } else {
+#pragma unroll
+        for (int c = 0; c < 32; ++c) a[c] = (c < valid) ? __bfloat162float(p[c]) : 0.f;
+    }
+}
+
+// One 32-column chunk of the tile for the 32 rows of one epilogue warp (this
+// lane's row m).  Values are rounded to bf16, staged per warp in shared memory
+// (sR: the rows, sT: the same block transposed) and written by TMA stores; the
+// column sums of a delta block (bias change) are read back from sT.
 template <int MODE>
-__device__ __forceinline__ void epilogue_chunk(const GemmArgs& g, int m, int n0, int split,
-                                               float (&v)[32], float& sse, bool row_ok) {
+__device__ __forceinline__ void epilogue_chunk(const GemmArgs& g, const CUtensorMap* map_r,
+                                               const CUtensorMap* map_t, int m, int m0, int n0,
+                                               int split, float (&v)[32], float& sse, bool row_ok,
+                                               bf16* sR, bf16* sT, float* colsum_slot) {
     const int N = g.N;
+    const int lane = threadIdx.x & 31;
     if (MODE == MODE_DW) {
         if (row_ok) {
             float* dst = g.gpart + ((size_t)split * g.M + m) * N + n0;
@@ -232,89 +267,91 @@ __device__ __forceinline__ void epilogue_chunk(const GemmArgs& g, int m, int n0,
         }
         return;
     }
-    // values that become bf16 outputs
-    float o[32];
+    const bool whole = (n0 + 32 <= N);
+    const int valid = min(32, N - n0);
+    const bool with_t = (MODE == MODE_FWD_OUT) && (g.aux != nullptr);
+    float vals[32];
     if (MODE == MODE_FWD || MODE == MODE_FWD_OUT) {
+        float b[32];
+        if (whole) {
 #pragma unroll
-        for (int c = 0; c < 32; ++c) {
-            const int n = min(n0 + c, N - 1);
-            o[c] = bf16_round(sigmoid_fast(v[c] + __ldg(g.bias + n)));
-        }
-    }
-    if (MODE == MODE_FWD) {
-        if (row_ok) {
-            bf16* dst = g.out + (size_t)m * g.ldo + n0;
-            if (n0 + 32 <= N) {
-#pragma unroll
-                for (int c = 0; c < 32; c += 8) {
-                    __align__(16) bf16 pk[8];
-#pragma unroll
-                    for (int q = 0; q < 8; ++q) pk[q] = __float2bfloat16_rn(o[c + q]);
-                    *reinterpret_cast<uint4*>(dst + c) = *reinterpret_cast<uint4*>(pk);
-                }
-            } else {
-                for (int c = 0; c < 32; ++c)
-                    if (n0 + c < N) dst[c] = __float2bfloat16_rn(o[c]);
-            }
-            if (g.out_t != nullptr) {
-                for (int c = 0; c < 32; ++c)
-                    if (n0 + c < N) g.out_t[(size_t)(n0 + c) * g.ldt + m] = __float2bfloat16_rn(o[c]);
-            }
-        }
-        return;
-    }
-    // delta-producing modes
-    float d[32];
-    if (MODE == MODE_FWD_OUT) {
-        if (row_ok && g.out != nullptr) {
-            bf16* dst = g.out + (size_t)m * g.ldo + n0;
-            for (int c = 0; c < 32; ++c)
-                if (n0 + c < N) dst[c] = __float2bfloat16_rn(o[c]);
-        }
-        if (g.aux == nullptr) return;
-#pragma unroll
-        for (int c = 0; c < 32; ++c) {
-            float t = 0.f;
-            if (row_ok && n0 + c < N) t = __bfloat162float(g.aux[(size_t)m * g.ld_aux + n0 + c]);
-            const float err = t - o[c];
-            const bool ok = row_ok && (n0 + c < N);
-            sse = ok ? fmaf(err, err, sse) : sse;
-            d[c] = ok ? bf16_round(err * o[c] * (1.f - o[c])) : 0.f;
-        }
-    } else {   // MODE_DX
-#pragma unroll
-        for (int c = 0; c < 32; ++c) {
-            float a = 0.f;
-            const bool ok = row_ok && (n0 + c < N);
-            if (ok) a = __bfloat162float(g.aux[(size_t)m * g.ld_aux + n0 + c]);
-            d[c] = ok ? bf16_round(v[c] * a * (1.f - a)) : 0.f;
-        }
-    }
-    bf16* drow = (MODE == MODE_FWD_OUT) ? g.out2 : g.out;
-    const int ldd = (MODE == MODE_FWD_OUT) ? g.ld2 : g.ldo;
-    if (row_ok && drow != nullptr) {
-        bf16* dst = drow + (size_t)m * ldd + n0;
-        if (n0 + 32 <= N) {
-#pragma unroll
-            for (int c = 0; c < 32; c += 8) {
-                __align__(16) bf16 pk[8];
-#pragma unroll
-                for (int q = 0; q < 8; ++q) pk[q] = __float2bfloat16_rn(d[c + q]);
-                *reinterpret_cast<uint4*>(dst + c) = *reinterpret_cast<uint4*>(pk);
+            for (int k = 0; k < 8; ++k) {
+                const float4 f = __ldg(reinterpret_cast<const float4*>(g.bias + n0) + k);
+                b[4 * k] = f.x;
+                b[4 * k + 1] = f.y;
+                b[4 * k + 2] = f.z;
+                b[4 * k + 3] = f.w;
             }
         } else {
-            for (int c = 0; c < 32; ++c)
-                if (n0 + c < N) dst[c] = __float2bfloat16_rn(d[c]);
+#pragma unroll
+            for (int c = 0; c < 32; ++c) b[c] = (c < valid) ? __ldg(g.bias + n0 + c) : 0.f;
+        }
+        float t[32];
+        if (with_t) load_row32(t, g.aux + (size_t)m * g.ld_aux + n0, whole && row_ok, row_ok ? valid : 0);
+#pragma unroll
+        for (int c = 0; c < 32; ++c) {
+            const bool ok = row_ok && (c < valid);
+            const float o = bf16_round(sigmoid_fast(v[c] + b[c]));
+            if (with_t) {
+                const float err = t[c] - o;
+                sse = ok ? fmaf(err, err, sse) : sse;
+                vals[c] = ok ? bf16_round(err * o * (1.f - o)) : 0.f;
+            } else {
+                vals[c] = ok ? o : 0.f;
+            }
+        }
+    } else {   // MODE_DX: delta_{l-1} = (delta_l W_l) a (1 - a)
+        float a[32];
+        load_row32(a, g.aux + (size_t)m * g.ld_aux + n0, whole && row_ok, row_ok ? valid : 0);
+#pragma unroll
+        for (int c = 0; c < 32; ++c) {
+            const bool ok = row_ok && (c < valid);
+            vals[c] = ok ? bf16_round(v[c] * a[c] * (1.f - a[c])) : 0.f;
         }
     }
-    if (row_ok) {
-        for (int c = 0; c < 32; ++c)
-            if (n0 + c < N) g.out_t[(size_t)(n0 + c) * g.ldt + m] = __float2bfloat16_rn(d[c]);
+    const bool has_r = (MODE == MODE_FWD) || (MODE == MODE_FWD_OUT) ||
+                       (MODE == MODE_DX && g.out != nullptr);
+    const bool has_t = (MODE == MODE_FWD && g.out_t != nullptr) || with_t || (MODE == MODE_DX);
+    if (has_r) {
+        uint4* dst = reinterpret_cast<uint4*>(sR + lane * 32);
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {
+            __align__(16) __nv_bfloat162 h[4];
+#pragma unroll
+            for (int q = 0; q < 4; ++q) h[q] = __floats2bfloat162_rn(vals[8 * k + 2 * q], vals[8 * k + 2 * q + 1]);
+            dst[k] = *reinterpret_cast<const uint4*>(h);
+        }
     }
-    // column sums of delta over this warp's 32 rows (bias change)
-    const int lane = threadIdx.x & 31;
-    reduce_scatter32(d, lane);
-    v[0] = d[0];   // lane c: sum of column n0 + c over the warp's rows
+    if (has_t) {
+#pragma unroll
+        for (int c = 0; c < 32; ++c) sT[c * 32 + lane] = __float2bfloat16_rn(vals[c]);
+    }
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+    __syncwarp();
+    if (lane == 0) {
+        if (has_r) tma_store_2d(map_r, sR, n0, m0);
+        if (has_t) tma_store_2d(map_t, sT, m0, n0);
+        asm volatile("cp.async.bulk.commit_group;" ::: "memory");
+    }
+    if (colsum_slot != nullptr) {
+        // lane c sums column c of the block over the warp's 32 rows
+        const uint4* col = reinterpret_cast<const uint4*>(sT + lane * 32);
+        float sum = 0.f;
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {
+            const uint4 u = col[k];
+            const __nv_bfloat162* h = reinterpret_cast<const __nv_bfloat162*>(&u);
+#pragma unroll
+            for (int q = 0; q < 4; ++q) {
+                const float2 f = __bfloat1622float2(h[q]);
+                sum += f.x;
+                sum += f.y;
+            }
+        }
+        colsum_slot[lane] = sum;
+    }
+    if (lane == 0) asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory");
+    __syncwarp();   // the staging blocks may be rewritten
 }
 
 // ------------------------------------------------------------ GEMM kernel
@@ -328,12 +365,14 @@ struct GemmCfg {
     // tile ring, then barriers and scratch
     static constexpr int kRingBytes = kStages * kStageBytes;
     static constexpr int kColsumBytes = 4 * BN * 4;
-    static constexpr int kSmemBytes = 1024 + kRingBytes + kColsumBytes + 256;
+    static constexpr int kStageOutBytes = 4 * 2 * 32 * 32 * 2;   // per epilogue warp: rows + transposed
+    static constexpr int kSmemBytes = 1024 + kRingBytes + kColsumBytes + kStageOutBytes + 256;
 };
 
 template <int BN, int MODE>
 __global__ void __launch_bounds__(kGemmThreads, 1)
     k_gemm(const __grid_constant__ CUtensorMap map_a, const __grid_constant__ CUtensorMap map_b,
+           const __grid_constant__ CUtensorMap map_r, const __grid_constant__ CUtensorMap map_t,
            GemmArgs g) {
     using Cfg = GemmCfg<BN, MODE>;
     constexpr int S = Cfg::kStages;
@@ -341,7 +380,9 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
     uint8_t* smem = reinterpret_cast<uint8_t*>(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
     uint8_t* ring = smem;
     float* colsum = reinterpret_cast<float*>(smem + Cfg::kRingBytes);   // [4][BN]
-    uint64_t* bars = reinterpret_cast<uint64_t*>(smem + Cfg::kRingBytes + Cfg::kColsumBytes);
+    bf16* stage_out = reinterpret_cast<bf16*>(smem + Cfg::kRingBytes + Cfg::kColsumBytes);
+    uint64_t* bars = reinterpret_cast<uint64_t*>(smem + Cfg::kRingBytes + Cfg::kColsumBytes +
+                                                 Cfg::kStageOutBytes);
     uint64_t* full = bars;              // [S]
     uint64_t* empty = bars + S;         // [S]
     uint64_t* tfull = bars + 2 * S;     // [2]
@@ -475,17 +516,20 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
             const bool row_ok = m < g.M;
             float sse = 0.f;
             const uint32_t tbase = tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(acc * BN);
+            const int m0 = mb * BM + q * 32;
+            bf16* sR = stage_out + ew * 2048;
+            bf16* sT = sR + 1024;
+            const bool want_colsum = (MODE == MODE_DX) || (MODE == MODE_FWD_OUT && g.aux != nullptr);
             for (int c0 = 0; c0 < BN; c0 += 32) {
                 const int n0 = nb * BN + c0;
                 float v[32];
                 tmem_ld32(tbase + (uint32_t)c0, v);
                 if (n0 >= g.N) {
-                    if (MODE == MODE_FWD_OUT || MODE == MODE_DX) colsum[ew * BN + c0 + lane] = 0.f;
+                    if (want_colsum) colsum[ew * BN + c0 + lane] = 0.f;
                     continue;
                 }
-                epilogue_chunk<MODE>(g, m, n0, split, v, sse, row_ok);
-                if (MODE == MODE_DX || (MODE == MODE_FWD_OUT && g.aux != nullptr))
-                    colsum[ew * BN + c0 + lane] = v[0];
+                epilogue_chunk<MODE>(g, &map_r, &map_t, m, m0, n0, split, v, sse, row_ok, sR, sT,
+                                     want_colsum ? colsum + ew * BN + c0 : nullptr);
             }
             // TMEM is free for the next accumulation into this buffer
             tc_fence_before();
@@ -515,6 +559,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
             }
         }
     }
+    if (warp >= 2 && lane == 0) asm volatile("cp.async.bulk.wait_group 0;" ::: "memory");
     tc_fence_before();
     __syncthreads();
     if (warp == 1) {
@@ -726,6 +771,19 @@ bool make_map(CUtensorMap* map, const void* base, int rows, int cols, int ld, in
     return r == CUDA_SUCCESS;
 }
 
+// Store map: [rows, cols] bf16, row pitch ld elements, 32 x 32 boxes, no swizzle.
+bool make_store_map(CUtensorMap* map, const void* base, int rows, int cols, int ld) {
+    cuuint64_t dims[2] = {(cuuint64_t)cols, (cuuint64_t)rows};
+    cuuint64_t strides[1] = {(cuuint64_t)ld * 2};
+    cuuint32_t box[2] = {32, 32};
+    cuuint32_t estr[2] = {1, 1};
+    CUresult r = g_encode(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims,
+                          strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                          CU_TENSOR_MAP_SWIZZLE_NONE, CU_TENSOR_MAP_L2_PROMOTION_NONE,
+                          CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    return r == CUDA_SUCCESS;
+}
+
 template <int BN, int MODE>
 cudaError_t gemm_setup() {
     return cudaFuncSetAttribute(k_gemm<BN, MODE>, cudaFuncAttributeMaxDynamicSharedMemorySize,
@@ -794,8 +852,8 @@ int pick_splits(int tiles, int kb_total, int num_sms, int cap_splits) {
 }
 
 template <int MODE>
-cudaError_t launch_gemm(const Bf16Net* b, const CUtensorMap& ma, const CUtensorMap& mb, GemmArgs g,
-                        cudaStream_t s) {
+cudaError_t launch_gemm(const Bf16Net* b, const CUtensorMap& ma, const CUtensorMap& mb,
+                        const CUtensorMap& mr, const CUtensorMap& mt, GemmArgs g, cudaStream_t s) {
     g.num_m = ceil_div(g.M, BM);
     g.num_n = ceil_div(g.N, kBN);
     g.kb_total = ceil_div(g.K, BK);
@@ -805,7 +863,7 @@ cudaError_t launch_gemm(const Bf16Net* b, const CUtensorMap& ma, const CUtensorM
     g.flags = b->flags;
     const int items = g.num_m * g.num_n * g.splits;
     const int grid = items < b->num_sms ? items : b->num_sms;
-    k_gemm<kBN, MODE><<<grid, kGemmThreads, GemmCfg<kBN, MODE>::kSmemBytes, s>>>(ma, mb, g);
+    k_gemm<kBN, MODE><<<grid, kGemmThreads, GemmCfg<kBN, MODE>::kSmemBytes, s>>>(ma, mb, mr, mt, g);
     return cudaGetLastError();
 }
 
@@ -831,16 +889,19 @@ cudaError_t run_forward(Bf16Net* b, const bf16* X, int B, const bf16* T, bf16* Y
         g.K = b->n[l - 1];
         g.bias = b->theta + b->boff[l];
         cudaError_t e;
+        CUtensorMap mr, mt;
         if (l < L) {
             g.out = b->act[l];
             g.ldo = b->n[l];
             g.out_t = b->actT[l];
             g.ldt = b->cap_pad;
-            e = launch_gemm<MODE_FWD>(b, ma, mb, g, s);
+            if (!make_store_map(&mr, g.out, B, b->n[l], b->n[l]) ||
+                !make_store_map(&mt, g.out_t, b->n[l], B, b->cap_pad))
+                return cudaErrorInvalidValue;
+            e = launch_gemm<MODE_FWD>(b, ma, mb, mr, mt, g, s);
         } else {
-            g.out = (Y != nullptr) ? Y : b->act[L];
-            g.ldo = b->n[L];
             if (T != nullptr) {
+                // training: the output deltas (rows and transposed) replace the outputs
                 g.aux = T;
                 g.ld_aux = b->n[L];
                 g.out2 = b->dlt[L];
@@ -849,8 +910,16 @@ cudaError_t run_forward(Bf16Net* b, const bf16* X, int B, const bf16* T, bf16* Y
                 g.ldt = b->cap_pad;
                 g.bias_part = b->bpart[L];
                 g.sse_part = b->sse_part;
+                if (!make_store_map(&mr, g.out2, B, b->n[L], b->n[L]) ||
+                    !make_store_map(&mt, g.out_t, b->n[L], B, b->cap_pad))
+                    return cudaErrorInvalidValue;
+            } else {
+                g.out = (Y != nullptr) ? Y : b->act[L];
+                g.ldo = b->n[L];
+                if (!make_store_map(&mr, g.out, B, b->n[L], b->n[L])) return cudaErrorInvalidValue;
+                mt = mr;
             }
-            e = launch_gemm<MODE_FWD_OUT>(b, ma, mb, g, s);
+            e = launch_gemm<MODE_FWD_OUT>(b, ma, mb, mr, mt, g, s);
         }
         if (e != cudaSuccess) return e;
     }
@@ -885,7 +954,14 @@ cudaError_t run_backward(Bf16Net* b, const bf16* X, int B, cudaStream_t s) {
         g.aux = b->act[l - 1];
         g.ld_aux = b->n[l - 1];
         g.bias_part = b->bpart[l - 1];
-        cudaError_t e = launch_gemm<MODE_DX>(b, ma, mb, g, s);
+        CUtensorMap mr, mt;
+        if (!make_store_map(&mt, g.out_t, b->n[l - 1], B, b->cap_pad)) return cudaErrorInvalidValue;
+        if (g.out != nullptr) {
+            if (!make_store_map(&mr, g.out, B, b->n[l - 1], b->n[l - 1])) return cudaErrorInvalidValue;
+        } else {
+            mr = mt;
+        }
+        cudaError_t e = launch_gemm<MODE_DX>(b, ma, mb, mr, mt, g, s);
         if (e != cudaSuccess) return e;
     }
     for (int l = 1; l <= L; ++l) {
@@ -902,7 +978,7 @@ cudaError_t run_backward(Bf16Net* b, const bf16* X, int B, cudaStream_t s) {
         g.splits = b->splits[l];
         const int tiles = ceil_div(g.M, BM) * ceil_div(g.N, kBN);
         g.splits = pick_splits(tiles, ceil_div(B, BK), b->num_sms, b->splits[l]);
-        cudaError_t e = launch_gemm<MODE_DW>(b, ma, mb, g, s);
+        cudaError_t e = launch_gemm<MODE_DW>(b, ma, mb, ma, ma, g, s);
         if (e != cudaSuccess) return e;
     }
     return cudaSuccess;

@@ -132,6 +132,17 @@ static void cl_make_carve(ClCarve& c, const int* n, int L, int C, int Pc, int R)
         c.soff[l] = c.slice;
         c.slice += c.wsz[l];
     }
+    for (int l = 1; l <= L; ++l) {   // offset of input unit j in its activation buffer
+        c.joff[l] = off;
+        off += (n[l - 1] + 4) & ~3;
+    }
+    for (int l = 2; l <= L; ++l) {   // column of input unit j in the partial-sum rows
+        c.sidx[l] = off;
+        off += (n[l - 1] + 3) & ~3;
+    }
+    // ---- per-chunk buffers; after the last chunk of a group they are dead and
+    // the staging ring of the copies' pooled changes reuses them
+    const int chunk0 = off;
     c.full[0] = off;          // the input chunk, row-major [Pc][pf0]
     off += Pc * c.pf[0];
     c.tin = off;              // targets of own output units, [Pc][nup_L]
@@ -148,14 +159,6 @@ static void cl_make_carve(ClCarve& c, const int* n, int L, int C, int Pc, int R)
         c.S[l] = off;
         off += Pc * C * c.nup[l - 1];
     }
-    for (int l = 1; l <= L; ++l) {   // offset of input unit j in its activation buffer
-        c.joff[l] = off;
-        off += (n[l - 1] + 4) & ~3;
-    }
-    for (int l = 2; l <= L; ++l) {   // column of input unit j in the partial-sum rows
-        c.sidx[l] = off;
-        off += (n[l - 1] + 3) & ~3;
-    }
     int red = 0;
     for (int l = 1; l <= L; ++l) {
         int ks = kThreads / Pc;
@@ -167,9 +170,9 @@ static void cl_make_carve(ClCarve& c, const int* n, int L, int C, int Pc, int R)
     }
     c.red = off;
     off += red;
-    c.stg = off;              // staging of R copies' pooled changes
-    off += R * c.slice;
-    c.total = off;
+    c.stg = chunk0;           // staging of R copies' pooled changes (aliases the chunk)
+    const int stg_end = chunk0 + R * c.slice;
+    c.total = off > stg_end ? off : stg_end;
 }
 
 namespace {
@@ -335,8 +338,13 @@ __global__ void __launch_bounds__(kThreads, 1)
                     for (int g = 0; g < nup; g += 8) {
                         float acc[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
                         if (p < pc) {
+                            if (l == 1) {
+#pragma unroll 4
+                                for (int j = j0; j < j1; ++j) fma8(acc, ip[j], W + j * nup + g);
+                            } else {
 #pragma unroll 2
-                            for (int j = j0; j < j1; ++j) fma8(acc, ip[jo[j]], W + j * nup + g);
+                                for (int j = j0; j < j1; ++j) fma8(acc, ip[jo[j]], W + j * nup + g);
+                            }
                         }
                         float* rp_ = red + (kq * Pc + p) * nup + g;
                         *reinterpret_cast<float4*>(rp_) = make_float4(acc[0], acc[1], acc[2], acc[3]);
@@ -521,9 +529,10 @@ __global__ void __launch_bounds__(kThreads, 1)
             cluster.sync();
             return;
         }
-        if (blockIdx.x == 0 && tid < 32) {
-            // error sum of the group: lane-strided partial sums, then a fixed
-            // butterfly, so that every run adds in the same order
+        if (blockIdx.x == gridDim.x - 1 && tid < 32) {
+            // error sum of the group, by the last CTA (the last rank owns the
+            // fewest units): lane-strided partial sums, then a fixed butterfly,
+            // so that every run adds in the same order
             const float* sp = a.sse_part + (size_t)buf * gridDim.x;
             float tot = 0.f;
             for (int k = tid; k < (int)gridDim.x; k += 32) tot += __ldcg(sp + k);
@@ -699,12 +708,13 @@ ClPlan cl_plan(const int* n, int L, int batch, int num_sms) {
         if (NC * C > num_sms) NC = num_sms / C;
         if (NC > kClMaxCopies) NC = kClMaxCopies;
         if (NC < 1) continue;
-        // chunk: the patterns a copy gets per group (a multiple of 32, at most
+        // chunk: the patterns a copy gets per group (a multiple of 8, at most
         // 256), shrunk until it fits; then as many staged copies as fit
         const int per = (batch + NC - 1) / NC;
-        int pc = ((per + 31) / 32) * 32;
+        int pc = ((per + 7) / 8) * 8;
         if (pc > 256) pc = 256;
-        while (pc > 32 && cl_smem_bytes(n, L, C, pc, 1) > kClSmemLimit) pc -= 32;
+        if (pc < 32) pc = 32;
+        while (pc > 32 && cl_smem_bytes(n, L, C, pc, 1) > kClSmemLimit) pc -= 8;
         int R = 1;
         while (R < NC && cl_smem_bytes(n, L, C, pc, R + 1) <= kClSmemLimit) ++R;
         ClPlan p;
