@@ -66,13 +66,6 @@ struct bp_net {
     unsigned* bar = nullptr;
     int* flags = nullptr;
     F32View view{};
-    // float32 cluster training kernel (weights resident in shared memory)
-    bool cl_ok = false;
-    ClArgs cl{};
-    float* gpart = nullptr;
-    float* cl_sse = nullptr;
-    int cl_plan_batch = -1;
-    ClPlan cl_last{};
     // bfloat16 path
     Bf16Net* bf = nullptr;
     // last forward, for bp_backward
@@ -101,8 +94,6 @@ void free_all(bp_net* net) {
     cudaFree(net->stage_X);
     cudaFree(net->stage_T);
     cudaFree(net->stage_sse);
-    cudaFree(net->gpart);
-    cudaFree(net->cl_sse);
     if (net->bf) bf16_destroy(net->bf);
 }
 
@@ -110,9 +101,6 @@ void refresh_view(bp_net* net) {
     net->view.lr = net->lr;
     net->view.momentum = net->momentum;
     net->view.grad_scale = net->grad_scale;
-    net->cl.lr = net->lr;
-    net->cl.momentum = net->momentum;
-    net->cl.grad_scale = net->grad_scale;
 }
 
 bp_status check_batch(const bp_net* net, int batch) {
@@ -172,7 +160,6 @@ bp_status bp_create(const int* sizes, int n_layers, float lr, float momentum, in
             std::lock_guard<std::mutex> lk(g_setup_mu);
             if (net->device < 64 && !g_f32_ready[net->device]) {
                 e = f32_setup(net->device);
-                if (e == cudaSuccess) e = cl_setup(net->device);
                 if (e != cudaSuccess) return bail(cuda_fail(e, "float32 kernel setup"));
                 g_f32_ready[net->device] = true;
             }
@@ -193,64 +180,18 @@ bp_status bp_create(const int* sizes, int n_layers, float lr, float momentum, in
 
     if (dtype == BP_F32) {
         F32View& v = net->view;
-        v.L = net->L;
-        v.cap = max_batch;
-        long long pos = 0, soff = 0;
-        int tiles = 0;
-        for (int l = 0; l <= net->L; ++l) v.n[l] = net->n[l];
-        v.tile0[0] = v.tile0[1] = 0;
-        for (int l = 1; l <= net->L; ++l) {
-            v.woff[l] = pos;
-            pos += (long long)net->n[l] * net->n[l - 1];
-            v.boff[l] = pos;
-            pos += net->n[l];
-            v.soff[l] = soff;
-            soff += (long long)max_batch * ((net->n[l] + 3) & ~3);
-            const int rows = (net->n[l] + 7) / 8, cols = (net->n[l - 1] + 1 + 31) / 32;
-            v.tcols[l] = cols;
-            v.tile0[l] = tiles;
-            tiles += rows * cols;
-            v.tile0[l + 1] = tiles;
-        }
-        e = cudaMalloc(&net->A, soff * sizeof(float));
-        if (e == cudaSuccess) e = cudaMalloc(&net->D, soff * sizeof(float));
+        f32_layout(v, net->n, net->L, max_batch);
+        e = cudaMalloc(&net->A, v.a_floats * sizeof(float));
+        if (e == cudaSuccess) e = cudaMalloc(&net->D, v.d_floats * sizeof(float));
         if (e == cudaSuccess) e = cudaMalloc(&net->sse_part, (size_t)net->num_sms * 4 * sizeof(float));
         if (e == cudaSuccess) e = cudaMalloc(&net->bar, 2 * sizeof(unsigned));
         if (e == cudaSuccess) e = cudaMalloc(&net->flags, sizeof(int));
         if (e != cudaSuccess) return bail(cuda_fail(e, "cudaMalloc(scratch)"));
         e = cudaMemset(net->bar, 0, 2 * sizeof(unsigned));
         if (e == cudaSuccess) e = cudaMemset(net->flags, 0, sizeof(int));
-        if (e == cudaSuccess) e = cudaMemset(net->A, 0, soff * sizeof(float));
-        if (e == cudaSuccess) e = cudaMemset(net->D, 0, soff * sizeof(float));
+        if (e == cudaSuccess) e = cudaMemset(net->A, 0, v.a_floats * sizeof(float));
+        if (e == cudaSuccess) e = cudaMemset(net->D, 0, v.d_floats * sizeof(float));
         if (e != cudaSuccess) return bail(cuda_fail(e, "cudaMemset(scratch)"));
-        // the cluster kernel, when the net's slices fit in shared memory
-        const ClPlan cp = cl_plan(net->n, net->L, max_batch, net->num_sms);
-        if (cp.ok) {
-            size_t gfl = 0;   // enough for either cluster size
-            for (int C = 8; C <= 16; C *= 2) {
-                const size_t f = (size_t)2 * (net->num_sms / C) * C * cl_slice_floats(net->n, net->L, C);
-                if (f > gfl) gfl = f;
-            }
-            e = cudaMalloc(&net->gpart, gfl * sizeof(float));
-            if (e == cudaSuccess) e = cudaMalloc(&net->cl_sse, (size_t)2 * net->num_sms * sizeof(float));
-            if (e != cudaSuccess) return bail(cuda_fail(e, "cudaMalloc(cluster scratch)"));
-            ClArgs& c = net->cl;
-            c.L = net->L;
-            for (int l = 0; l <= net->L; ++l) c.n[l] = net->n[l];
-            for (int l = 1; l <= net->L; ++l) {
-                c.woff[l] = v.woff[l];
-                c.boff[l] = v.boff[l];
-            }
-            c.P = P;
-            c.theta = net->theta;
-            c.V = net->V;
-            c.G = net->G;
-            c.gpart = net->gpart;
-            c.sse_part = net->cl_sse;
-            c.bar = net->bar;
-            c.flags = net->flags;
-            net->cl_ok = true;
-        }
         v.theta = net->theta;
         v.V = net->V;
         v.G = net->G;
@@ -362,7 +303,7 @@ bp_status bp_backward(bp_net* net, const void* d_T, int batch, float* d_sse, voi
         const F32Plan plan = f32_plan(net->view, batch, net->num_sms);
         BP_CUDA(f32_backward(net->view, (const float*)net->fwd_X, (const float*)d_T, batch, d_sse,
                              plan, s),
-                "bp_backward");
+                "bp_backward");   // the forward kept its inputs in scratch
     } else {
         BP_CUDA(bf16_backward(net->bf, net->fwd_X, d_T, batch, d_sse, net->g_dirty, s),
                 "bp_backward");
@@ -387,24 +328,10 @@ static bp_status run_epoch(bp_net* net, const void* d_X, const void* d_T, int n_
                            int minibatch, float* d_sse, cudaStream_t s) {
     const int n_steps = (int)(((long long)n_patterns + minibatch - 1) / minibatch);
     if (net->dtype == BP_F32) {
-        if (net->cl_ok && net->cl_plan_batch != minibatch) {
-            net->cl_last = cl_plan(net->n, net->L, minibatch, net->num_sms);
-            net->cl_plan_batch = minibatch;
-        }
-        // the cluster kernel when each copy's share of a group fits in one chunk
-        // (its cost per chunk is mostly latency); otherwise the persistent kernel
-        const bool use_cl = net->cl_ok && net->cl_last.ok &&
-                            (long long)net->cl_last.Pc * net->cl_last.NC >= minibatch;
-        if (use_cl) {
-            BP_CUDA(f32_train_cluster(net->cl, (const float*)d_X, (const float*)d_T, n_patterns,
-                                      minibatch, n_steps, d_sse, net->g_dirty, net->cl_last, s),
-                    "training launch");
-        } else {
-            const F32Plan plan = f32_plan(net->view, minibatch, net->num_sms);
-            BP_CUDA(f32_train(net->view, (const float*)d_X, (const float*)d_T, n_patterns,
-                              minibatch, n_steps, d_sse, net->g_dirty, plan, s),
-                    "training launch");
-        }
+        const F32Plan plan = f32_plan(net->view, minibatch, net->num_sms);
+        BP_CUDA(f32_train(net->view, (const float*)d_X, (const float*)d_T, n_patterns, minibatch,
+                          n_steps, d_sse, net->g_dirty, plan, s),
+                "training launch");
     } else {
         BP_CUDA(bf16_train(net->bf, d_X, d_T, n_patterns, minibatch, d_sse, net->lr, net->momentum,
                            net->grad_scale, net->g_dirty, s),

@@ -1,22 +1,24 @@
-// float32 back-propagation step on CUDA cores (FFMA), for nets whose per-pattern
-// activations fit in shared memory (the NETtalk-sized nets of Section 6.3).
+// float32 back-propagation step on CUDA cores (FFMA).
 //
 // One training step over a group of B patterns runs in two phases:
 //
-//   pattern phase (case-parallel, Section 4.1): each CTA takes groups of PG
-//     patterns and runs the whole net on them -- forward pass (Section 3),
+//   pattern phase (case-parallel, Section 4.1): every CTA first copies all the
+//     weights into its shared memory with one bulk copy (they fit for the
+//     NETtalk-sized nets of Section 6.3; larger nets read them from L2), then
+//     runs the whole net on its share of the patterns: forward pass (Section 3),
 //     output delta (t-o)o(1-o) with the summed squared error, hidden deltas
 //     (W^T delta) h(1-h) for every hidden layer and none for the inputs
-//     (Section 6.1).  Activations and deltas live in shared memory; weights
-//     stream from L2.  Dot products are summed as a binary tree across the
-//     warp (Section 10.3).
+//     (Section 6.1).  Dot products are summed as a binary tree across the
+//     warp (Section 10.3).  Activations (with a trailing 1 for the bias input)
+//     and deltas go to scratch rows aligned to 16 bytes.
 //
-//   weight phase (one CTA per 8 x 32 tile of weights, Section 5's "bundle"
-//     processed over the whole group of cases): the pooled change
-//     G[j,i] = sum_p delta[p,j] a[p,i] over all B patterns (Sections 3, 4.1),
-//     then either G += tile (bp_backward) or directly the momentum update of
-//     Section 6.2.1 (training launches), so the pooled change never leaves
-//     registers.
+//   weight phase (Section 5's "bundle" of weights processed over the whole
+//     group of cases): one CTA per 8 x 32 tile of [W_l | b_l] stages the
+//     group's deltas and activations through shared memory with 16-byte
+//     cp.async, sums delta[p,j] a[p,i] over all patterns with 4-wide register
+//     blocking (Sections 3, 4.1), then either accumulates into G (bp_backward)
+//     or applies the momentum update of Section 6.2.1 at once (training), so the
+//     pooled change never goes to memory.
 //
 // A training launch is a persistent cooperative kernel that loops over any
 // number of groups with a grid barrier between the phases; every wait in the
@@ -31,14 +33,16 @@
 namespace bp {
 namespace {
 
-constexpr int kThreads = 256;
+constexpr int kThreads = 512;
 constexpr int kWarps = kThreads / 32;
-constexpr int kTJ = 8;            // weight-tile rows (output units)
-constexpr int kTI = 32;           // weight-tile columns (input units + bias)
-constexpr int kPC = 256;          // patterns per staged chunk in the weight phase
-constexpr size_t kGradSmem = 2ull * kPC * (kTJ + kTI) * sizeof(float);
+constexpr int kTU = 8;            // weight-tile rows (output units)
+constexpr int kTJ = 32;           // weight-tile columns (inputs; the bias is the last input)
+constexpr int kPC = 256;          // patterns per staged chunk of the weight phase
+constexpr int kPS = kThreads / (kTJ * kTU / 4);   // pattern splits per tile (8)
+constexpr int kChunkFloats = kPC * (kTU + kTJ);
+constexpr size_t kGradFloats = 2 * kChunkFloats + kPS * kTU * kTJ;
 
-constexpr unsigned long long kWaitNs = 2000000000ull;   // 2 s per barrier wait
+constexpr unsigned long long kWaitNs = 2000000000ull;   // 2 s per wait
 constexpr unsigned kWaitIters = 1u << 26;
 
 // ------------------------------------------------------------ small helpers
@@ -63,6 +67,9 @@ __device__ __forceinline__ unsigned long long global_ns() {
     asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
     return t;
 }
+__device__ __forceinline__ uint32_t smem_u32(const void* p) {
+    return (uint32_t)__cvta_generic_to_shared(p);
+}
 
 // Sense-reversing grid barrier for a cooperative launch.  Returns false (in
 // every thread of the CTA) if the wait ran out; the caller must then return.
@@ -71,6 +78,7 @@ __device__ bool grid_barrier(unsigned* bar, int* flags) {
     __syncthreads();
     if (threadIdx.x == 0) {
         int ok = 1;
+        __threadfence();
         const unsigned gen = ld_acquire(bar + 1);
         const unsigned prev = atom_add_acq_rel(bar, 1u);
         if (prev == gridDim.x - 1) {
@@ -86,7 +94,7 @@ __device__ bool grid_barrier(unsigned* bar, int* flags) {
                     ok = 0;
                     break;
                 }
-                if (it > 256) __nanosleep(64);
+                if (it > 512) __nanosleep(32);
             }
         }
         s_ok = ok;
@@ -132,13 +140,63 @@ __device__ __forceinline__ void reduce_scatter32(float (&v)[32], int lane) {
     }
 }
 
+// ------------------------------------------------------------ weights in shared memory
+__device__ __forceinline__ void mbar_init1(uint64_t* bar) {
+    if (threadIdx.x == 0) {
+        asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(smem_u32(bar)) : "memory");
+        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    }
+    __syncthreads();
+}
+
+// Copies theta[0, P) into shared memory Ws (one bulk copy for the 16-byte
+// aligned part, plain loads for the tail).  Bounded wait on the mbarrier.
+__device__ void stage_weights(const float* theta, long long P, float* Ws, uint64_t* bar,
+                              unsigned& phase, int* flags) {
+    const long long P16 = P & ~3LL;
+    if (threadIdx.x == 0 && P16 > 0) {
+        asm volatile("fence.proxy.async.global;" ::: "memory");
+        asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+        const unsigned bytes = (unsigned)(P16 * 4);
+        asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_u32(bar)),
+                     "r"(bytes)
+                     : "memory");
+        asm volatile(
+            "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::
+                "r"(smem_u32(Ws)),
+            "l"(theta), "r"(bytes), "r"(smem_u32(bar))
+            : "memory");
+    }
+    for (long long k = P16 + threadIdx.x; k < P; k += kThreads) Ws[k] = __ldcg(theta + k);
+    if (P16 > 0) {
+        unsigned done = 0;
+        const unsigned long long t0 = global_ns();
+        for (unsigned it = 0;; ++it) {
+            asm volatile(
+                "{\n\t.reg .pred p;\n\t"
+                "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+                "selp.u32 %0, 1, 0, p;\n\t}"
+                : "=r"(done)
+                : "r"(smem_u32(bar)), "r"(phase)
+                : "memory");
+            if (done) break;
+            if ((it & 255u) == 255u && global_ns() - t0 > kWaitNs) {
+                if (threadIdx.x == 0) atomicOr(flags, kFlagTimeout);
+                break;
+            }
+        }
+        phase ^= 1u;
+    }
+    __syncthreads();
+}
+
 // ------------------------------------------------------------ pattern phase
 // Forward through one layer for PG patterns held in shared memory:
 // out[p][j] = sigma(sum_i W[j][i] in[p][i] + b[j]).  A warp owns 32/PG units at
 // a time; lanes stride over the inputs.
 template <int PG>
-__device__ void forward_layer(const float* __restrict__ W, const float* __restrict__ b,
-                              int n_in, int n_out, const float* s_in, float* s_out) {
+__device__ void forward_layer(const float* W, const float* b, int n_in, int n_out, const float* s_in,
+                              float* s_out) {
     constexpr int UJ = 32 / PG;
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     for (int j0 = warp * UJ; j0 < n_out; j0 += kWarps * UJ) {
@@ -152,7 +210,7 @@ __device__ void forward_layer(const float* __restrict__ W, const float* __restri
 #pragma unroll
             for (int u = 0; u < UJ; ++u) {
                 const int j = min(j0 + u, n_out - 1);   // rows past the end are discarded
-                const float w = __ldcg(W + (size_t)j * n_in + i);
+                const float w = W[(size_t)j * n_in + i];
 #pragma unroll
                 for (int p = 0; p < PG; ++p) acc[u * PG + p] = fmaf(w, a[p], acc[u * PG + p]);
             }
@@ -160,17 +218,19 @@ __device__ void forward_layer(const float* __restrict__ W, const float* __restri
         reduce_scatter32(acc, lane);
         const int u = lane / PG, p = lane % PG;
         const int j = j0 + u;
-        if (j < n_out) s_out[p * n_out + j] = sigmoid_f(acc[0] + __ldcg(b + j));
+        if (j < n_out) s_out[p * n_out + j] = sigmoid_f(acc[0] + b[j]);
     }
 }
 
-// Runs the pattern phase for this CTA's groups of `B` patterns.
+// Runs the pattern phase for this CTA's share of the group's B patterns
+// (patterns [blockIdx.x*B/gridDim.x, (blockIdx.x+1)*B/gridDim.x), PG at a time).
+//   Wb: the weights (shared memory copy or global theta)
 //   do_fwd: forward pass from X (else the activations are reloaded from scratch)
 //   do_bwd: deltas against T, written to scratch
 //   Y: if not null, the outputs are copied there ([B, n_L] packed)
 // Returns this CTA's summed squared error (valid in thread 0).
 template <int PG>
-__device__ float pattern_phase(const F32View& v, const float* __restrict__ X,
+__device__ float pattern_phase(const F32View& v, const float* Wb, const float* __restrict__ X,
                                const float* __restrict__ T, int B, bool do_fwd, bool do_bwd,
                                float* __restrict__ Y, float* smem) {
     const int L = v.L;
@@ -182,10 +242,10 @@ __device__ float pattern_phase(const F32View& v, const float* __restrict__ X,
         for (int l = 1; l <= L; ++l) { sd[l] = off; off += PG * v.n[l]; }
     }
     float sse = 0.f;
-    const int ngroups = (B + PG - 1) / PG;
-    for (int g = blockIdx.x; g < ngroups; g += gridDim.x) {
-        const int p0 = g * PG;
-        const int np = min(PG, B - p0);
+    const int q_lo = (int)((long long)B * blockIdx.x / gridDim.x);
+    const int q_hi = (int)((long long)B * (blockIdx.x + 1) / gridDim.x);
+    for (int p0 = q_lo; p0 < q_hi; p0 += PG) {
+        const int np = min(PG, q_hi - p0);
         if (do_fwd) {
             const int n0 = v.n[0];
             for (int e = tid; e < PG * n0; e += kThreads) {
@@ -194,17 +254,19 @@ __device__ float pattern_phase(const F32View& v, const float* __restrict__ X,
             }
             __syncthreads();
             for (int l = 1; l <= L; ++l) {
-                forward_layer<PG>(v.theta + v.woff[l], v.theta + v.boff[l], v.n[l - 1], v.n[l],
-                                  smem + sa[l - 1], smem + sa[l]);
+                forward_layer<PG>(Wb + v.woff[l], Wb + v.boff[l], v.n[l - 1], v.n[l], smem + sa[l - 1],
+                                  smem + sa[l]);
                 __syncthreads();
             }
-            for (int l = 1; l <= L; ++l) {
-                const int n = v.n[l];
-                const int pitch = (n + 3) & ~3;
-                float* dst = v.A + v.soff[l];
-                for (int e = tid; e < PG * n; e += kThreads) {
-                    const int p = e / n, i = e - p * n;
-                    if (p < np) dst[(size_t)(p0 + p) * pitch + i] = smem[sa[l] + e];
+            // activation rows (a trailing 1 is the true unit's input, zeros pad the row)
+            for (int l = 0; l <= L; ++l) {
+                const int n = v.n[l], pitch = v.apitch[l];
+                float* dst = v.A + v.aoff[l];
+                for (int e = tid; e < PG * pitch; e += kThreads) {
+                    const int p = e / pitch, i = e - p * pitch;
+                    if (p < np)
+                        dst[(size_t)(p0 + p) * pitch + i] =
+                            (i < n) ? smem[sa[l] + p * n + i] : (i == n ? 1.f : 0.f);
                 }
             }
             if (Y != nullptr) {
@@ -216,9 +278,8 @@ __device__ float pattern_phase(const F32View& v, const float* __restrict__ X,
             }
         } else {
             for (int l = 1; l <= L; ++l) {
-                const int n = v.n[l];
-                const int pitch = (n + 3) & ~3;
-                const float* src = v.A + v.soff[l];
+                const int n = v.n[l], pitch = v.apitch[l];
+                const float* src = v.A + v.aoff[l];
                 for (int e = tid; e < PG * n; e += kThreads) {
                     const int p = e / n, i = e - p * n;
                     smem[sa[l] + e] = (p < np) ? __ldcg(src + (size_t)(p0 + p) * pitch + i) : 0.f;
@@ -244,13 +305,14 @@ __device__ float pattern_phase(const F32View& v, const float* __restrict__ X,
             // hidden deltas, output side first; no delta for the input layer
             for (int l = L - 1; l >= 1; --l) {
                 const int n = v.n[l], nn = v.n[l + 1];
-                const float* Wn = v.theta + v.woff[l + 1];
+                const float* Wn = Wb + v.woff[l + 1];
                 for (int i = tid; i < n; i += kThreads) {
                     float acc[PG];
 #pragma unroll
                     for (int p = 0; p < PG; ++p) acc[p] = 0.f;
+#pragma unroll 2
                     for (int j = 0; j < nn; ++j) {
-                        const float w = __ldcg(Wn + (size_t)j * n + i);
+                        const float w = Wn[(size_t)j * n + i];
 #pragma unroll
                         for (int p = 0; p < PG; ++p)
                             acc[p] = fmaf(smem[sd[l + 1] + p * nn + j], w, acc[p]);
@@ -264,12 +326,11 @@ __device__ float pattern_phase(const F32View& v, const float* __restrict__ X,
                 __syncthreads();
             }
             for (int l = 1; l <= L; ++l) {
-                const int n = v.n[l];
-                const int pitch = (n + 3) & ~3;
-                float* dst = v.D + v.soff[l];
-                for (int e = tid; e < PG * n; e += kThreads) {
-                    const int p = e / n, i = e - p * n;
-                    if (p < np) dst[(size_t)(p0 + p) * pitch + i] = smem[sd[l] + e];
+                const int n = v.n[l], pitch = v.dpitch[l];
+                float* dst = v.D + v.doff[l];
+                for (int e = tid; e < PG * pitch; e += kThreads) {
+                    const int p = e / pitch, i = e - p * pitch;
+                    if (p < np) dst[(size_t)(p0 + p) * pitch + i] = (i < n) ? smem[sd[l] + p * n + i] : 0.f;
                 }
             }
         }
@@ -279,147 +340,126 @@ __device__ float pattern_phase(const F32View& v, const float* __restrict__ X,
 }
 
 // ------------------------------------------------------------ weight phase
-__device__ __forceinline__ void cp_async4(float* dst, const float* src) {
-    const unsigned d = (unsigned)__cvta_generic_to_shared(dst);
-    asm volatile("cp.async.ca.shared.global [%0], [%1], 4;" ::"r"(d), "l"(src) : "memory");
-}
 __device__ __forceinline__ void cp_async16(float* dst, const float* src) {
-    const unsigned d = (unsigned)__cvta_generic_to_shared(dst);
-    asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(d), "l"(src) : "memory");
+    asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(smem_u32(dst)), "l"(src) : "memory");
 }
 __device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
 template <int N>
 __device__ __forceinline__ void cp_async_wait() { asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory"); }
 
-// Stage patterns [c*kPC, c*kPC + pc) of a weight tile: sD[pp][0..8) = delta rows
-// j0.., sA[pp][0..32) = activation columns i0.. (zeros past the ends).
-__device__ void stage_chunk(float* sD, float* sA, const float* Dl, int pitch_out, int n_out, int j0,
-                            const float* Ain, int pitch_in, int n_in, int i0, bool in_is_x,
-                            int p0, int pc) {
-    const int tid = threadIdx.x;
-    // deltas: two float4 per pattern row (scratch rows are 16-byte aligned)
-    for (int e = tid; e < kPC * 2; e += kThreads) {
-        const int pp = e >> 1, q = (e & 1) * 4;
-        float* dst = sD + pp * kTJ + q;
-        if (pp < pc && j0 + q < pitch_out) {
-            cp_async16(dst, Dl + (size_t)(p0 + pp) * pitch_out + j0 + q);
+// Stage patterns [p0, p0 + pc) of a tile: Ds[pp][0..8) = delta columns u0..,
+// As[pp][0..32) = activation columns j0.. (rows are 16-byte aligned; zeros past
+// the ends of a row and past pc).
+__device__ void stage_tile(float* Ds, float* As, const float* Dl, int dpitch, int u0,
+                           const float* Al, int apitch, int j0, int p0, int pc) {
+    for (int e = threadIdx.x; e < kPC * 10; e += kThreads) {
+        const int pp = e / 10, q = e - pp * 10;
+        float* dst;
+        const float* src;
+        bool ok;
+        if (q < 2) {
+            dst = Ds + pp * kTU + q * 4;
+            ok = pp < pc && u0 + q * 4 < dpitch;
+            src = Dl + (size_t)(p0 + pp) * dpitch + u0 + q * 4;
         } else {
-            dst[0] = dst[1] = dst[2] = dst[3] = 0.f;
+            const int c = (q - 2) * 4;
+            dst = As + pp * kTJ + c;
+            ok = pp < pc && j0 + c < apitch;
+            src = Al + (size_t)(p0 + pp) * apitch + j0 + c;
+        }
+        if (ok) {
+            cp_async16(dst, src);
+        } else {
+            *reinterpret_cast<float4*>(dst) = make_float4(0.f, 0.f, 0.f, 0.f);
         }
     }
-    if (!in_is_x) {
-        for (int e = tid; e < kPC * 8; e += kThreads) {
-            const int pp = e >> 3, q = (e & 7) * 4;
-            float* dst = sA + pp * kTI + q;
-            if (pp < pc && i0 + q < pitch_in) {
-                cp_async16(dst, Ain + (size_t)(p0 + pp) * pitch_in + i0 + q);
-            } else {
-                dst[0] = dst[1] = dst[2] = dst[3] = 0.f;
-            }
-        }
-    } else {
-        // caller's input rows: any pitch, read-only for the whole launch
-        for (int e = tid; e < kPC * kTI; e += kThreads) {
-            const int pp = e >> 5, q = e & 31;
-            float* dst = sA + pp * kTI + q;
-            if (pp < pc && i0 + q < n_in) {
-                cp_async4(dst, Ain + (size_t)(p0 + pp) * n_in + i0 + q);
-            } else {
-                *dst = 0.f;
-            }
-        }
-    }
-    (void)n_out;
 }
 
-// Pooled change of every weight over the B patterns of the group, then either
-// accumulate into G (fused == false) or apply the update directly.
-__device__ void weight_phase(const F32View& v, const float* __restrict__ X, int B, bool fused,
-                             bool fold_g, float* smem) {
+// Pooled change of every weight (and bias: the last input column is the true
+// unit's 1) over the B patterns of the group, then either accumulate into G
+// (fused == false) or apply the update directly.
+__device__ void weight_phase(const F32View& v, int B, bool fused, bool fold_g, float* smem) {
     const int tid = threadIdx.x;
-    const int tj = tid >> 5, ti = tid & 31;
-    float* sD[2] = {smem, smem + kPC * kTJ};
-    float* sA[2] = {smem + 2 * kPC * kTJ, smem + 2 * kPC * kTJ + kPC * kTI};
+    // thread = (pattern split ps, 4 output units uq, input column j)
+    const int ps = tid / (kTJ * kTU / 4), r = tid - ps * (kTJ * kTU / 4);
+    const int uq = r / kTJ, j = r - uq * kTJ;
+    float* red = smem + 2 * kChunkFloats;   // [kPS][kTU][kTJ]
     const int L = v.L;
     const int ntiles = v.tile0[L + 1];
     const int nchunks = (B + kPC - 1) / kPC;
+    constexpr int kPer = kPC / kPS;   // patterns per thread per chunk
     for (int t = blockIdx.x; t < ntiles; t += gridDim.x) {
         int l = 1;
         while (t >= v.tile0[l + 1]) ++l;
         const int lt = t - v.tile0[l];
-        const int jb = lt / v.tcols[l], ib = lt - jb * v.tcols[l];
+        const int tb = lt / v.tcols[l], cb = lt - tb * v.tcols[l];
         const int n_in = v.n[l - 1], n_out = v.n[l];
-        const int j0 = jb * kTJ, i0 = ib * kTI;
-        const bool in_is_x = (l == 1);
-        const float* Ain = in_is_x ? X : v.A + v.soff[l - 1];
-        const int pitch_in = in_is_x ? n_in : ((n_in + 3) & ~3);
-        const float* Dl = v.D + v.soff[l];
-        const int pitch_out = (n_out + 3) & ~3;
-        const int i = i0 + ti, j = j0 + tj;
-        const bool bias_col = (i == n_in);
-
-        float acc0 = 0.f, acc1 = 0.f, acc2 = 0.f, acc3 = 0.f;
-        stage_chunk(sD[0], sA[0], Dl, pitch_out, n_out, j0, Ain, pitch_in, n_in, i0, in_is_x, 0,
-                    min(kPC, B));
+        const int u0 = tb * kTU, j0 = cb * kTJ;
+        const float* Dl = v.D + v.doff[l];
+        const float* Al = v.A + v.aoff[l - 1];
+        float acc[4] = {0.f, 0.f, 0.f, 0.f};
+        stage_tile(smem, smem + kPC * kTU, Dl, v.dpitch[l], u0, Al, v.apitch[l - 1], j0, 0,
+                   min(kPC, B));
         cp_async_commit();
         for (int c = 0; c < nchunks; ++c) {
             if (c + 1 < nchunks) {
                 const int p0 = (c + 1) * kPC;
-                stage_chunk(sD[(c + 1) & 1], sA[(c + 1) & 1], Dl, pitch_out, n_out, j0, Ain,
-                            pitch_in, n_in, i0, in_is_x, p0, min(kPC, B - p0));
+                float* nb = smem + ((c + 1) & 1) * kChunkFloats;
+                stage_tile(nb, nb + kPC * kTU, Dl, v.dpitch[l], u0, Al, v.apitch[l - 1], j0, p0,
+                           min(kPC, B - p0));
                 cp_async_commit();
                 cp_async_wait<1>();
             } else {
                 cp_async_wait<0>();
             }
             __syncthreads();
-            const float* d = sD[c & 1] + tj;
-            const float* a = sA[c & 1] + ti;
-            const int pc = min(kPC, B - c * kPC);
-            int pp = 0;
-            if (!bias_col) {
-                for (; pp + 4 <= pc; pp += 4) {
-                    acc0 = fmaf(d[(pp + 0) * kTJ], a[(pp + 0) * kTI], acc0);
-                    acc1 = fmaf(d[(pp + 1) * kTJ], a[(pp + 1) * kTI], acc1);
-                    acc2 = fmaf(d[(pp + 2) * kTJ], a[(pp + 2) * kTI], acc2);
-                    acc3 = fmaf(d[(pp + 3) * kTJ], a[(pp + 3) * kTI], acc3);
-                }
-                for (; pp < pc; ++pp) acc0 = fmaf(d[pp * kTJ], a[pp * kTI], acc0);
-            } else {
-                // the true unit's activation is 1
-                for (; pp + 4 <= pc; pp += 4) {
-                    acc0 += d[(pp + 0) * kTJ];
-                    acc1 += d[(pp + 1) * kTJ];
-                    acc2 += d[(pp + 2) * kTJ];
-                    acc3 += d[(pp + 3) * kTJ];
-                }
-                for (; pp < pc; ++pp) acc0 += d[pp * kTJ];
+            const float* Ds = smem + (c & 1) * kChunkFloats;
+            const float* As = Ds + kPC * kTU;
+            const int pp0 = ps * kPer;
+#pragma unroll 4
+            for (int k = 0; k < kPer; ++k) {
+                const int pp = pp0 + k;
+                const float4 d = *reinterpret_cast<const float4*>(Ds + pp * kTU + uq * 4);
+                const float a = As[pp * kTJ + j];
+                acc[0] = fmaf(d.x, a, acc[0]);
+                acc[1] = fmaf(d.y, a, acc[1]);
+                acc[2] = fmaf(d.z, a, acc[2]);
+                acc[3] = fmaf(d.w, a, acc[3]);
             }
             __syncthreads();
         }
-        const float g = (acc0 + acc1) + (acc2 + acc3);
-        if (j < n_out && i <= n_in) {
-            const long long idx = bias_col ? v.boff[l] + j : v.woff[l] + (long long)j * n_in + i;
-            if (!fused) {
-                v.G[idx] += g;
-            } else {
-                float gt = g;
-                if (fold_g) {
-                    gt += v.G[idx];
-                    v.G[idx] = 0.f;
+#pragma unroll
+        for (int k = 0; k < 4; ++k) red[(ps * kTU + uq * 4 + k) * kTJ + j] = acc[k];
+        __syncthreads();
+        if (tid < kTU * kTJ) {
+            const int u = tid / kTJ, jj = tid - u * kTJ;
+            float g = 0.f;
+#pragma unroll
+            for (int s = 0; s < kPS; ++s) g += red[(s * kTU + u) * kTJ + jj];
+            const int uu = u0 + u, ii = j0 + jj;
+            if (uu < n_out && ii <= n_in) {
+                const long long idx = (ii < n_in) ? v.woff[l] + (long long)uu * n_in + ii : v.boff[l] + uu;
+                if (!fused) {
+                    v.G[idx] += g;
+                } else {
+                    if (fold_g) {
+                        g += v.G[idx];
+                        v.G[idx] = 0.f;
+                    }
+                    const float vel = v.lr * v.grad_scale * g + v.momentum * v.V[idx];
+                    v.V[idx] = vel;
+                    v.theta[idx] += vel;
                 }
-                const float vel = v.lr * v.grad_scale * gt + v.momentum * v.V[idx];
-                v.V[idx] = vel;
-                v.theta[idx] += vel;
             }
         }
+        __syncthreads();
     }
 }
 
-// Error sum of the group by the first warp of CTA 0: lane-strided partial sums
-// then a fixed butterfly (the same order on every run).
+// Error sum of the group by the first warp of the last CTA: lane-strided
+// partial sums then a fixed butterfly (the same order on every run).
 __device__ void reduce_sse(const F32View& v, int nparts, float* sse_out) {
-    if (blockIdx.x == 0 && threadIdx.x < 32) {
+    if (blockIdx.x == gridDim.x - 1 && threadIdx.x < 32) {
         float s = 0.f;
         for (int c = threadIdx.x; c < nparts; c += 32) s += __ldcg(v.sse_part + c);
         s = warp_sum(s);
@@ -431,30 +471,47 @@ __device__ void reduce_sse(const F32View& v, int nparts, float* sse_out) {
 }
 
 // ------------------------------------------------------------ kernels
-template <int PG>
-__global__ void __launch_bounds__(kThreads) k_forward(F32View v, const float* X, int B, float* Y) {
-    extern __shared__ float smem[];
-    pattern_phase<PG>(v, X, nullptr, B, true, false, Y, smem);
+// WS: the weights are copied into shared memory (else read from global memory).
+template <int PG, bool WS>
+__global__ void __launch_bounds__(kThreads, 1) k_forward(F32View v, const float* X, int B, float* Y) {
+    extern __shared__ __align__(16) float smem[];
+    __shared__ __align__(8) uint64_t s_bar;
+    unsigned phase = 0;
+    if (WS) {
+        mbar_init1(&s_bar);
+        stage_weights(v.theta, v.P, smem, &s_bar, phase, v.flags);
+        pattern_phase<PG>(v, smem, X, nullptr, B, true, false, Y, smem + v.wsm);
+    } else {
+        pattern_phase<PG>(v, v.theta, X, nullptr, B, true, false, Y, smem);
+    }
 }
 
-template <int PG>
-__global__ void __launch_bounds__(kThreads) k_deltas(F32View v, const float* T, int B) {
-    extern __shared__ float smem[];
-    const float e = pattern_phase<PG>(v, nullptr, T, B, false, true, nullptr, smem);
+template <int PG, bool WS>
+__global__ void __launch_bounds__(kThreads, 1) k_deltas(F32View v, const float* T, int B) {
+    extern __shared__ __align__(16) float smem[];
+    __shared__ __align__(8) uint64_t s_bar;
+    unsigned phase = 0;
+    float e;
+    if (WS) {
+        mbar_init1(&s_bar);
+        stage_weights(v.theta, v.P, smem, &s_bar, phase, v.flags);
+        e = pattern_phase<PG>(v, smem, nullptr, T, B, false, true, nullptr, smem + v.wsm);
+    } else {
+        e = pattern_phase<PG>(v, v.theta, nullptr, T, B, false, true, nullptr, smem);
+    }
     if (threadIdx.x == 0) v.sse_part[blockIdx.x] = e;
 }
 
-__global__ void __launch_bounds__(kThreads)
-    k_accumulate(F32View v, const float* X, int B, int nparts, float* sse_out) {
-    extern __shared__ float smem[];
+__global__ void __launch_bounds__(kThreads, 1)
+    k_accumulate(F32View v, int B, int nparts, float* sse_out) {
+    extern __shared__ __align__(16) float smem[];
     reduce_sse(v, nparts, sse_out);
-    weight_phase(v, X, B, false, false, smem);
+    weight_phase(v, B, false, false, smem);
 }
 
-__global__ void __launch_bounds__(kThreads) k_update(F32View v, long long n) {
+__global__ void __launch_bounds__(256) k_update(F32View v, long long n) {
     const float a = v.lr * v.grad_scale, m = v.momentum;
-    for (long long k = blockIdx.x * (long long)kThreads + threadIdx.x; k < n;
-         k += (long long)gridDim.x * kThreads) {
+    for (long long k = blockIdx.x * 256LL + threadIdx.x; k < n; k += (long long)gridDim.x * 256) {
         const float vel = a * v.G[k] + m * v.V[k];
         v.V[k] = vel;
         v.theta[k] += vel;
@@ -462,42 +519,58 @@ __global__ void __launch_bounds__(kThreads) k_update(F32View v, long long n) {
     }
 }
 
-template <int PG>
-__global__ void __launch_bounds__(kThreads)
-    k_train(F32View v, const float* X, const float* T, int n_patterns, int minibatch,
-            int n_steps, float* sse_out, int fold_g) {
-    extern __shared__ float smem[];
+template <int PG, bool WS>
+__global__ void __launch_bounds__(kThreads, 1)
+    k_train(F32View v, const float* X, const float* T, int n_patterns, int minibatch, int n_steps,
+            float* sse_out, int fold_g) {
+    extern __shared__ __align__(16) float smem[];
+    __shared__ __align__(8) uint64_t s_bar;
     // A latched timeout means an earlier launch left the barrier half-way; do
     // nothing until bp_check() has cleared the latch and reset the barrier.
     if (__ldcg(v.flags) & kFlagTimeout) return;
+    unsigned phase = 0;
+    mbar_init1(&s_bar);
     const int n0 = v.n[0], nL = v.n[v.L];
     for (int s = 0; s < n_steps; ++s) {
         const long long p0 = (long long)s * minibatch;
         const int B = (int)min((long long)minibatch, (long long)n_patterns - p0);
         const float* Xs = X + p0 * n0;
         const float* Ts = T + p0 * nL;
-        const float e = pattern_phase<PG>(v, Xs, Ts, B, true, true, nullptr, smem);
+        float e;
+        if (WS) {
+            stage_weights(v.theta, v.P, smem, &s_bar, phase, v.flags);
+            e = pattern_phase<PG>(v, smem, Xs, Ts, B, true, true, nullptr, smem + v.wsm);
+        } else {
+            e = pattern_phase<PG>(v, v.theta, Xs, Ts, B, true, true, nullptr, smem);
+        }
         if (threadIdx.x == 0) v.sse_part[blockIdx.x] = e;
         if (!grid_barrier(v.bar, v.flags)) return;
         reduce_sse(v, gridDim.x, sse_out != nullptr ? sse_out + s : nullptr);
-        weight_phase(v, Xs, B, true, fold_g != 0 && s == 0, smem);
+        weight_phase(v, B, true, fold_g != 0 && s == 0, smem);
         if (s + 1 < n_steps) {
             if (!grid_barrier(v.bar, v.flags)) return;
         }
     }
 }
 
+template <int PG, bool WS>
+cudaError_t set_smem_attr_ws(size_t bytes) {
+    cudaError_t e;
+    if ((e = cudaFuncSetAttribute(k_forward<PG, WS>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                  (int)bytes)) != cudaSuccess)
+        return e;
+    if ((e = cudaFuncSetAttribute(k_deltas<PG, WS>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                  (int)bytes)) != cudaSuccess)
+        return e;
+    return cudaFuncSetAttribute(k_train<PG, WS>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                (int)bytes);
+}
+
 template <int PG>
 cudaError_t set_smem_attr(size_t bytes) {
-    cudaError_t e;
-    if ((e = cudaFuncSetAttribute(k_forward<PG>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                  (int)bytes)) != cudaSuccess)
-        return e;
-    if ((e = cudaFuncSetAttribute(k_deltas<PG>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                  (int)bytes)) != cudaSuccess)
-        return e;
-    return cudaFuncSetAttribute(k_train<PG>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                (int)bytes);
+    cudaError_t e = set_smem_attr_ws<PG, true>(bytes);
+    if (e != cudaSuccess) return e;
+    return set_smem_attr_ws<PG, false>(bytes);
 }
 
 }  // namespace
@@ -508,12 +581,50 @@ cudaError_t set_smem_attr(size_t bytes) {
 constexpr size_t kStaticSmemReserve = 1024;
 constexpr size_t kSmemLimit = 227 * 1024 - kStaticSmemReserve;
 
-size_t f32_smem_bytes(const int* n, int L, int pg) {
+long long f32_layout(F32View& v, const int* n, int L, int cap) {
+    v.L = L;
+    v.cap = cap;
+    long long pos = 0, a = 0, d = 0;
+    int tiles = 0;
+    for (int l = 0; l <= L; ++l) v.n[l] = n[l];
+    v.tile0[0] = v.tile0[1] = 0;
+    for (int l = 0; l <= L; ++l) {
+        v.apitch[l] = (n[l] + 1 + 3) & ~3;
+        v.aoff[l] = a;
+        a += (long long)cap * v.apitch[l];
+    }
+    for (int l = 1; l <= L; ++l) {
+        v.woff[l] = pos;
+        pos += (long long)n[l] * n[l - 1];
+        v.boff[l] = pos;
+        pos += n[l];
+        v.dpitch[l] = (n[l] + 3) & ~3;
+        v.doff[l] = d;
+        d += (long long)cap * v.dpitch[l];
+        const int rows = (n[l] + kTU - 1) / kTU, cols = (n[l - 1] + 1 + kTJ - 1) / kTJ;
+        v.tcols[l] = cols;
+        v.tile0[l] = tiles;
+        tiles += rows * cols;
+        v.tile0[l + 1] = tiles;
+    }
+    v.P = pos;
+    v.wsm = (int)((pos + 3) & ~3LL);
+    v.a_floats = a;
+    v.d_floats = d;
+    return a + d;
+}
+
+static size_t pattern_floats(const int* n, int L, int pg) {
     size_t units = 0;
     for (int l = 0; l <= L; ++l) units += (size_t)n[l];
     for (int l = 1; l <= L; ++l) units += (size_t)n[l];
-    const size_t pattern = units * (size_t)pg * sizeof(float);
-    return pattern > kGradSmem ? pattern : kGradSmem;
+    return units * (size_t)pg;
+}
+
+size_t f32_smem_bytes(const int* n, int L, int pg) {
+    const size_t grad = kGradFloats * sizeof(float);
+    const size_t pat = pattern_floats(n, L, pg) * sizeof(float);
+    return pat > grad ? pat : grad;
 }
 
 int f32_max_pg(const int* n, int L) {
@@ -533,7 +644,7 @@ cudaError_t f32_setup(int device) {
     if ((e = set_smem_attr<4>(kSmemLimit)) != cudaSuccess) return e;
     if ((e = set_smem_attr<8>(kSmemLimit)) != cudaSuccess) return e;
     return cudaFuncSetAttribute(k_accumulate, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                (int)kGradSmem);
+                                (int)(kGradFloats * sizeof(float)));
 }
 
 F32Plan f32_plan(const F32View& v, int batch, int num_sms) {
@@ -544,46 +655,56 @@ F32Plan f32_plan(const F32View& v, int batch, int num_sms) {
     while (pg < want && pg < maxpg) pg *= 2;
     p.pg = pg;
     p.grid = num_sms;
-    p.smem = f32_smem_bytes(v.n, v.L, pg);
+    // weights in shared memory when they fit beside the pattern buffers
+    const size_t wbytes = (size_t)v.wsm * sizeof(float);
+    const size_t pat = pattern_floats(v.n, v.L, pg) * sizeof(float);
+    const size_t grad = kGradFloats * sizeof(float);
+    p.w_in_smem = (wbytes + pat <= kSmemLimit) ? 1 : 0;
+    const size_t need = p.w_in_smem ? wbytes + pat : pat;
+    p.smem = need > grad ? need : grad;
     return p;
 }
 
 cudaError_t f32_forward(const F32View& v, const float* X, int batch, float* Y, const F32Plan& plan,
                         cudaStream_t s) {
-    const int groups = (batch + plan.pg - 1) / plan.pg;
-    const int grid = groups < plan.grid ? groups : plan.grid;
+#define BP_FWD(PG)                                                                        \
+    (plan.w_in_smem ? (k_forward<PG, true><<<plan.grid, kThreads, plan.smem, s>>>(v, X, batch, Y)) \
+                    : (k_forward<PG, false><<<plan.grid, kThreads, plan.smem, s>>>(v, X, batch, Y)))
     switch (plan.pg) {
-        case 1: k_forward<1><<<grid, kThreads, plan.smem, s>>>(v, X, batch, Y); break;
-        case 2: k_forward<2><<<grid, kThreads, plan.smem, s>>>(v, X, batch, Y); break;
-        case 4: k_forward<4><<<grid, kThreads, plan.smem, s>>>(v, X, batch, Y); break;
-        default: k_forward<8><<<grid, kThreads, plan.smem, s>>>(v, X, batch, Y); break;
+        case 1: BP_FWD(1); break;
+        case 2: BP_FWD(2); break;
+        case 4: BP_FWD(4); break;
+        default: BP_FWD(8); break;
     }
+#undef BP_FWD
     return cudaGetLastError();
 }
 
-cudaError_t f32_backward(const F32View& v, const float* X, const float* T, int batch,
+cudaError_t f32_backward(const F32View& v, const float* /*X*/, const float* T, int batch,
                          float* sse_out, const F32Plan& plan, cudaStream_t s) {
-    const int groups = (batch + plan.pg - 1) / plan.pg;
-    const int grid = groups < plan.grid ? groups : plan.grid;
+#define BP_DEL(PG)                                                                      \
+    (plan.w_in_smem ? (k_deltas<PG, true><<<plan.grid, kThreads, plan.smem, s>>>(v, T, batch)) \
+                    : (k_deltas<PG, false><<<plan.grid, kThreads, plan.smem, s>>>(v, T, batch)))
     switch (plan.pg) {
-        case 1: k_deltas<1><<<grid, kThreads, plan.smem, s>>>(v, T, batch); break;
-        case 2: k_deltas<2><<<grid, kThreads, plan.smem, s>>>(v, T, batch); break;
-        case 4: k_deltas<4><<<grid, kThreads, plan.smem, s>>>(v, T, batch); break;
-        default: k_deltas<8><<<grid, kThreads, plan.smem, s>>>(v, T, batch); break;
+        case 1: BP_DEL(1); break;
+        case 2: BP_DEL(2); break;
+        case 4: BP_DEL(4); break;
+        default: BP_DEL(8); break;
     }
+#undef BP_DEL
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return e;
     const int tiles = v.tile0[v.L + 1];
     const int ggrid = tiles < plan.grid ? tiles : plan.grid;
-    k_accumulate<<<ggrid, kThreads, kGradSmem, s>>>(v, X, batch, grid, sse_out);
+    k_accumulate<<<ggrid, kThreads, kGradFloats * sizeof(float), s>>>(v, batch, plan.grid, sse_out);
     return cudaGetLastError();
 }
 
 cudaError_t f32_update(const F32View& v, long long n_params, cudaStream_t s) {
-    long long blocks = (n_params + kThreads - 1) / kThreads;
+    long long blocks = (n_params + 255) / 256;
     if (blocks > 4096) blocks = 4096;
     if (blocks < 1) blocks = 1;
-    k_update<<<(int)blocks, kThreads, 0, s>>>(v, n_params);
+    k_update<<<(int)blocks, 256, 0, s>>>(v, n_params);
     return cudaGetLastError();
 }
 
@@ -595,11 +716,12 @@ cudaError_t f32_train(const F32View& v, const float* X, const float* T, int n_pa
     void* args[] = {(void*)&vv, (void*)&X, (void*)&T, (void*)&n_patterns, (void*)&minibatch,
                     (void*)&n_steps, (void*)&sse_out, (void*)&fold};
     const void* fn;
+    const bool ws = plan.w_in_smem != 0;
     switch (plan.pg) {
-        case 1: fn = (const void*)k_train<1>; break;
-        case 2: fn = (const void*)k_train<2>; break;
-        case 4: fn = (const void*)k_train<4>; break;
-        default: fn = (const void*)k_train<8>; break;
+        case 1: fn = ws ? (const void*)k_train<1, true> : (const void*)k_train<1, false>; break;
+        case 2: fn = ws ? (const void*)k_train<2, true> : (const void*)k_train<2, false>; break;
+        case 4: fn = ws ? (const void*)k_train<4, true> : (const void*)k_train<4, false>; break;
+        default: fn = ws ? (const void*)k_train<8, true> : (const void*)k_train<8, false>; break;
     }
     return cudaLaunchCooperativeKernel(fn, dim3(plan.grid), dim3(kThreads), args, plan.smem, s);
 }

@@ -102,29 +102,11 @@ extern "C" bp_status bp_train_epoch_noalloc(const int* layer_sizes, int n_layers
     if (st != BP_OK) return st;
 
     // scratch layout (floats, each part 16-byte aligned):
-    // [error word, pad][barrier x2, pad][per-CTA error sums][A rows][D rows]
+    // [error word, pad][barrier x2, pad][per-CTA error sums][activation rows][delta rows]
     F32View v{};
-    v.L = L;
-    v.cap = minibatch;
-    long long pos = 0, soff = 0;
-    int tiles = 0;
-    for (int l = 0; l <= L; ++l) v.n[l] = layer_sizes[l];
-    v.tile0[0] = v.tile0[1] = 0;
-    for (int l = 1; l <= L; ++l) {
-        v.woff[l] = pos;
-        pos += (long long)layer_sizes[l] * layer_sizes[l - 1];
-        v.boff[l] = pos;
-        pos += layer_sizes[l];
-        v.soff[l] = soff;
-        soff += (long long)minibatch * ((layer_sizes[l] + 3) & ~3);
-        const int rows = (layer_sizes[l] + 7) / 8, cols = (layer_sizes[l - 1] + 1 + 31) / 32;
-        v.tcols[l] = cols;
-        v.tile0[l] = tiles;
-        tiles += rows * cols;
-        v.tile0[l + 1] = tiles;
-    }
+    const long long soff = f32_layout(v, layer_sizes, L, minibatch);
     const long long head = 4 + 4 + (((long long)sms + 3) & ~3LL);
-    const long long need = head + 2 * soff;
+    const long long need = head + soff;
     if (need > (long long)kNoallocScratchFloats) {
         snprintf(msg, sizeof msg,
                  "bp_train_epoch_noalloc: these sizes and minibatch %d need %lld bytes of scratch; "
@@ -137,7 +119,7 @@ extern "C" bp_status bp_train_epoch_noalloc(const int* layer_sizes, int n_layers
     v.bar = reinterpret_cast<unsigned*>(base + 4);
     v.sse_part = base + 8;
     v.A = base + head;
-    v.D = base + head + soff;
+    v.D = base + head + v.a_floats;
     v.theta = d_theta;
     v.V = d_V;
     v.G = nullptr;   // nothing pending: the launch never reads G
