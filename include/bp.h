@@ -163,9 +163,9 @@ bp_status bp_check(bp_net* net, void* stream);
  *   Scratch (activations, deltas, barrier, error word) lives in one static
  *   device array of 8 MiB, which every GPU that loads the library holds until the
  *   process exits.  Sizes whose scratch exceeds it are rejected with
- *   BP_EINVAL; the scratch takes 4 * (16 + SMs + minibatch * (sum over
+ *   BP_EINVAL; the scratch takes 4 * (8 + roundup4(SMs) + minibatch * (sum over
  *   l = 0..L of roundup4(n_l + 1) + sum over l = 1..L of roundup4(n_l))) bytes
- *   (for 203-120-26 a minibatch of up to about 4,100 patterns fits).
+ *   (for 203-120-26 on 152 SMs a minibatch of up to 4,160 patterns fits).
  *   The first call on a device looks up the array's device address and sets
  *   kernel attributes; make that first call before any stream capture.  All
  *   calls on a device share the array and find the previous call's contents:

@@ -184,10 +184,10 @@ bp_status bp_create(const int* sizes, int n_layers, float lr, float momentum, in
         e = cudaMalloc(&net->A, v.a_floats * sizeof(float));
         if (e == cudaSuccess) e = cudaMalloc(&net->D, v.d_floats * sizeof(float));
         if (e == cudaSuccess) e = cudaMalloc(&net->sse_part, (size_t)net->num_sms * 4 * sizeof(float));
-        if (e == cudaSuccess) e = cudaMalloc(&net->bar, 2 * sizeof(unsigned));
+        if (e == cudaSuccess) e = cudaMalloc(&net->bar, (size_t)bp::kBarWords * sizeof(unsigned));
         if (e == cudaSuccess) e = cudaMalloc(&net->flags, sizeof(int));
         if (e != cudaSuccess) return bail(cuda_fail(e, "cudaMalloc(scratch)"));
-        e = cudaMemset(net->bar, 0, 2 * sizeof(unsigned));
+        e = cudaMemset(net->bar, 0, (size_t)bp::kBarWords * sizeof(unsigned));
         if (e == cudaSuccess) e = cudaMemset(net->flags, 0, sizeof(int));
         if (e == cudaSuccess) e = cudaMemset(net->A, 0, v.a_floats * sizeof(float));
         if (e == cudaSuccess) e = cudaMemset(net->D, 0, v.d_floats * sizeof(float));
@@ -367,7 +367,8 @@ bp_status bp_check(bp_net* net, void* stream) {
     BP_CUDA(cudaMemcpy(&flags, net->flags, sizeof(int), cudaMemcpyDeviceToHost), "bp_check");
     if (flags == 0) return BP_OK;
     BP_CUDA(cudaMemset(net->flags, 0, sizeof(int)), "bp_check");
-    if (net->bar) BP_CUDA(cudaMemset(net->bar, 0, 2 * sizeof(unsigned)), "bp_check");
+    if (net->bar)
+        BP_CUDA(cudaMemset(net->bar, 0, (size_t)bp::kBarWords * sizeof(unsigned)), "bp_check");
     if (flags & kFlagTimeout)
         return fail(BP_ETIMEOUT, "a bounded device-side wait ran out; the launch stopped early");
     return fail(BP_ENONFINITE, "the summed squared error of a group was not finite");

@@ -53,15 +53,6 @@ __device__ __forceinline__ unsigned ld_acquire(const unsigned* p) {
     asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
     return v;
 }
-__device__ __forceinline__ void st_release(unsigned* p, unsigned v) {
-    asm volatile("st.release.gpu.global.u32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
-}
-__device__ __forceinline__ unsigned atom_add_acq_rel(unsigned* p, unsigned v) {
-    unsigned old;
-    asm volatile("atom.acq_rel.gpu.global.add.u32 %0, [%1], %2;"
-                 : "=r"(old) : "l"(p), "r"(v) : "memory");
-    return old;
-}
 __device__ __forceinline__ unsigned long long global_ns() {
     unsigned long long t;
     asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
@@ -71,36 +62,35 @@ __device__ __forceinline__ uint32_t smem_u32(const void* p) {
     return (uint32_t)__cvta_generic_to_shared(p);
 }
 
-// Sense-reversing grid barrier for a cooperative launch.  Returns false (in
-// every thread of the CTA) if the wait ran out; the caller must then return.
-__device__ bool grid_barrier(unsigned* bar, int* flags) {
-    __shared__ int s_ok;
+// Grid barrier for a cooperative launch.  bar[1] counts arrivals over every
+// launch on the net; bar[0] holds its value at the end of the previous launch.
+// Barrier k of a launch completes when the count reaches bar[0] + k * grid:
+// thread 0 of each CTA adds its arrival with a fire-and-forget release
+// reduction and then polls the count (no CTA has to relay a release).  The
+// wait is bounded; on a timeout the error word latches kFlagTimeout and the
+// function returns false in every thread of the CTA (the caller must then
+// return).  Counts compare modulo 2^32.
+__device__ __forceinline__ bool count_reached(unsigned v, unsigned target) {
+    return (int)(v - target) >= 0;
+}
+__device__ bool grid_barrier(unsigned* bar, unsigned target, int* flags) {
     __syncthreads();
+    int ok = 1;
     if (threadIdx.x == 0) {
-        int ok = 1;
         __threadfence();
-        const unsigned gen = ld_acquire(bar + 1);
-        const unsigned prev = atom_add_acq_rel(bar, 1u);
-        if (prev == gridDim.x - 1) {
-            atomicExch(bar, 0u);
-            st_release(bar + 1, gen + 1u);
-        } else {
-            const unsigned long long t0 = global_ns();
-            unsigned it = 0;
-            while (ld_acquire(bar + 1) == gen) {
-                ++it;
-                if (it > kWaitIters || ((it & 63u) == 0 && global_ns() - t0 > kWaitNs)) {
-                    atomicOr(flags, kFlagTimeout);
-                    ok = 0;
-                    break;
-                }
-                if (it > 512) __nanosleep(32);
+        asm volatile("red.release.gpu.global.add.u32 [%0], %1;" ::"l"(bar + 1), "r"(1u) : "memory");
+        const unsigned long long t0 = global_ns();
+        unsigned it = 0;
+        while (!count_reached(ld_acquire(bar + 1), target)) {
+            ++it;
+            if (it > kWaitIters || ((it & 63u) == 0 && global_ns() - t0 > kWaitNs)) {
+                atomicOr(flags, kFlagTimeout);
+                ok = 0;
+                break;
             }
         }
-        s_ok = ok;
     }
-    __syncthreads();
-    return s_ok != 0;
+    return __syncthreads_and(ok) != 0;
 }
 
 __device__ __forceinline__ float warp_sum(float x) {
@@ -191,6 +181,57 @@ __device__ void stage_weights(const float* theta, long long P, float* Ws, uint64
 }
 
 // ------------------------------------------------------------ pattern phase
+__device__ __forceinline__ void cp_async16(float* dst, const float* src) {
+    asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(smem_u32(dst)), "l"(src) : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
+template <int N>
+__device__ __forceinline__ void cp_async_wait() { asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory"); }
+__device__ __forceinline__ void cp_async4(float* dst, const float* src) {
+    asm volatile("cp.async.ca.shared.global [%0], [%1], 4;" ::"r"(smem_u32(dst)), "l"(src) : "memory");
+}
+
+// Shared memory: the weights (WS) at the bottom, the pattern buffers above
+// them; the weight phase reuses the bottom kGradFloats floats for its tiles.
+template <bool WS>
+__device__ __forceinline__ float* pattern_base(const F32View& v, float* smem) {
+    return WS ? smem + v.wsm : smem;
+}
+
+// Offset of the target rows inside the pattern buffers (after the activation
+// and delta rows of PG patterns).
+template <int PG>
+__device__ __forceinline__ int target_offset(const F32View& v) {
+    int units = 0;
+    for (int l = 0; l <= v.L; ++l) units += v.n[l];
+    for (int l = 1; l <= v.L; ++l) units += v.n[l];
+    return PG * units;
+}
+
+// Issues the copies of the input rows (into sx, [PG][n0]) and target rows (into
+// st, [PG][nL]) of patterns [p0, p0 + np); rows past np are zeroed.  One
+// cp.async group; the caller waits for it before use.  (Issuing them one group
+// ahead, to land during the barrier and the weight phase, measured no faster.)
+template <int PG>
+__device__ void load_rows(const float* X, const float* T, int n0, int nL, int p0, int np, float* sx,
+                          float* st) {
+    if (X != nullptr) {
+        for (int e = threadIdx.x; e < PG * n0; e += kThreads) {
+            const int p = e / n0, i = e - p * n0;
+            if (p < np) cp_async4(sx + e, X + (size_t)(p0 + p) * n0 + i);
+            else sx[e] = 0.f;
+        }
+    }
+    if (T != nullptr) {
+        for (int e = threadIdx.x; e < PG * nL; e += kThreads) {
+            const int p = e / nL, k = e - p * nL;
+            if (p < np) cp_async4(st + e, T + (size_t)(p0 + p) * nL + k);
+            else st[e] = 0.f;
+        }
+    }
+    cp_async_commit();
+}
+
 // Forward through one layer for PG patterns held in shared memory:
 // out[p][j] = sigma(sum_i W[j][i] in[p][i] + b[j]).  A warp owns 32/PG units at
 // a time; lanes stride over the inputs.
@@ -235,24 +276,24 @@ __device__ float pattern_phase(const F32View& v, const float* Wb, const float* _
                                float* __restrict__ Y, float* smem) {
     const int L = v.L;
     const int tid = threadIdx.x;
+    const int n0 = v.n[0], nL = v.n[L];
     int sa[BP_MAX_SIZES], sd[BP_MAX_SIZES];
     {
         int off = 0;
         for (int l = 0; l <= L; ++l) { sa[l] = off; off += PG * v.n[l]; }
         for (int l = 1; l <= L; ++l) { sd[l] = off; off += PG * v.n[l]; }
     }
+    const int st = target_offset<PG>(v);
     float sse = 0.f;
     const int q_lo = (int)((long long)B * blockIdx.x / gridDim.x);
     const int q_hi = (int)((long long)B * (blockIdx.x + 1) / gridDim.x);
     for (int p0 = q_lo; p0 < q_hi; p0 += PG) {
         const int np = min(PG, q_hi - p0);
+        load_rows<PG>(do_fwd ? X : nullptr, do_bwd ? T : nullptr, n0, nL, p0, np, smem + sa[0],
+                      smem + st);
+        cp_async_wait<0>();
+        __syncthreads();
         if (do_fwd) {
-            const int n0 = v.n[0];
-            for (int e = tid; e < PG * n0; e += kThreads) {
-                const int p = e / n0, i = e - p * n0;
-                smem[sa[0] + e] = (p < np) ? __ldg(X + (size_t)(p0 + p) * n0 + i) : 0.f;
-            }
-            __syncthreads();
             for (int l = 1; l <= L; ++l) {
                 forward_layer<PG>(Wb + v.woff[l], Wb + v.boff[l], v.n[l - 1], v.n[l], smem + sa[l - 1],
                                   smem + sa[l]);
@@ -289,13 +330,12 @@ __device__ float pattern_phase(const F32View& v, const float* Wb, const float* _
         }
         if (do_bwd) {
             // output delta and error sum (Section 3, fn. 5)
-            const int nL = v.n[L];
             for (int e = tid; e < PG * nL; e += kThreads) {
-                const int p = e / nL, k = e - p * nL;
+                const int p = e / nL;
                 float d = 0.f;
                 if (p < np) {
                     const float o = smem[sa[L] + e];
-                    const float err = __ldg(T + (size_t)(p0 + p) * nL + k) - o;
+                    const float err = smem[st + e] - o;
                     sse = fmaf(err, err, sse);
                     d = err * o * (1.f - o);
                 }
@@ -340,12 +380,6 @@ __device__ float pattern_phase(const F32View& v, const float* Wb, const float* _
 }
 
 // ------------------------------------------------------------ weight phase
-__device__ __forceinline__ void cp_async16(float* dst, const float* src) {
-    asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(smem_u32(dst)), "l"(src) : "memory");
-}
-__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
-template <int N>
-__device__ __forceinline__ void cp_async_wait() { asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory"); }
 
 // Stage patterns [p0, p0 + pc) of a tile: Ds[pp][0..8) = delta columns u0..,
 // As[pp][0..32) = activation columns j0.. (rows are 16-byte aligned; zeros past
@@ -480,9 +514,9 @@ __global__ void __launch_bounds__(kThreads, 1) k_forward(F32View v, const float*
     if (WS) {
         mbar_init1(&s_bar);
         stage_weights(v.theta, v.P, smem, &s_bar, phase, v.flags);
-        pattern_phase<PG>(v, smem, X, nullptr, B, true, false, Y, smem + v.wsm);
+        pattern_phase<PG>(v, smem, X, nullptr, B, true, false, Y, pattern_base<true>(v, smem));
     } else {
-        pattern_phase<PG>(v, v.theta, X, nullptr, B, true, false, Y, smem);
+        pattern_phase<PG>(v, v.theta, X, nullptr, B, true, false, Y, pattern_base<false>(v, smem));
     }
 }
 
@@ -495,9 +529,9 @@ __global__ void __launch_bounds__(kThreads, 1) k_deltas(F32View v, const float* 
     if (WS) {
         mbar_init1(&s_bar);
         stage_weights(v.theta, v.P, smem, &s_bar, phase, v.flags);
-        e = pattern_phase<PG>(v, smem, nullptr, T, B, false, true, nullptr, smem + v.wsm);
+        e = pattern_phase<PG>(v, smem, nullptr, T, B, false, true, nullptr, pattern_base<true>(v, smem));
     } else {
-        e = pattern_phase<PG>(v, v.theta, nullptr, T, B, false, true, nullptr, smem);
+        e = pattern_phase<PG>(v, v.theta, nullptr, T, B, false, true, nullptr, pattern_base<false>(v, smem));
     }
     if (threadIdx.x == 0) v.sse_part[blockIdx.x] = e;
 }
@@ -530,7 +564,11 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (__ldcg(v.flags) & kFlagTimeout) return;
     unsigned phase = 0;
     mbar_init1(&s_bar);
+    // arrival count at the end of the previous launch; barrier k waits for
+    // base + k * grid arrivals
+    unsigned target = __ldcg(v.bar);
     const int n0 = v.n[0], nL = v.n[v.L];
+    float* pat = pattern_base<WS>(v, smem);
     for (int s = 0; s < n_steps; ++s) {
         const long long p0 = (long long)s * minibatch;
         const int B = (int)min((long long)minibatch, (long long)n_patterns - p0);
@@ -539,18 +577,21 @@ __global__ void __launch_bounds__(kThreads, 1)
         float e;
         if (WS) {
             stage_weights(v.theta, v.P, smem, &s_bar, phase, v.flags);
-            e = pattern_phase<PG>(v, smem, Xs, Ts, B, true, true, nullptr, smem + v.wsm);
+            e = pattern_phase<PG>(v, smem, Xs, Ts, B, true, true, nullptr, pat);
         } else {
-            e = pattern_phase<PG>(v, v.theta, Xs, Ts, B, true, true, nullptr, smem);
+            e = pattern_phase<PG>(v, v.theta, Xs, Ts, B, true, true, nullptr, pat);
         }
         if (threadIdx.x == 0) v.sse_part[blockIdx.x] = e;
-        if (!grid_barrier(v.bar, v.flags)) return;
+        if (!grid_barrier(v.bar, target += gridDim.x, v.flags)) return;
         reduce_sse(v, gridDim.x, sse_out != nullptr ? sse_out + s : nullptr);
         weight_phase(v, B, true, fold_g != 0 && s == 0, smem);
         if (s + 1 < n_steps) {
-            if (!grid_barrier(v.bar, v.flags)) return;
+            if (!grid_barrier(v.bar, target += gridDim.x, v.flags)) return;
         }
     }
+    // every CTA has passed a barrier, so every CTA has read bar[0]: publish the
+    // count for the next launch
+    if (blockIdx.x == 0 && threadIdx.x == 0) v.bar[0] = target;
 }
 
 template <int PG, bool WS>
@@ -618,13 +659,15 @@ static size_t pattern_floats(const int* n, int L, int pg) {
     size_t units = 0;
     for (int l = 0; l <= L; ++l) units += (size_t)n[l];
     for (int l = 1; l <= L; ++l) units += (size_t)n[l];
+    units += (size_t)n[L];   // target rows
     return units * (size_t)pg;
 }
 
+// Without the weights in shared memory: the pattern buffers and the
+// weight-phase tiles share the same bytes.
 size_t f32_smem_bytes(const int* n, int L, int pg) {
-    const size_t grad = kGradFloats * sizeof(float);
-    const size_t pat = pattern_floats(n, L, pg) * sizeof(float);
-    return pat > grad ? pat : grad;
+    const size_t pat = pattern_floats(n, L, pg);
+    return (pat > (size_t)kGradFloats ? pat : (size_t)kGradFloats) * sizeof(float);
 }
 
 int f32_max_pg(const int* n, int L) {
@@ -655,13 +698,12 @@ F32Plan f32_plan(const F32View& v, int batch, int num_sms) {
     while (pg < want && pg < maxpg) pg *= 2;
     p.pg = pg;
     p.grid = num_sms;
-    // weights in shared memory when they fit beside the pattern buffers
-    const size_t wbytes = (size_t)v.wsm * sizeof(float);
-    const size_t pat = pattern_floats(v.n, v.L, pg) * sizeof(float);
-    const size_t grad = kGradFloats * sizeof(float);
-    p.w_in_smem = (wbytes + pat <= kSmemLimit) ? 1 : 0;
-    const size_t need = p.w_in_smem ? wbytes + pat : pat;
-    p.smem = need > grad ? need : grad;
+    // weights in shared memory when they fit below the pattern buffers
+    const size_t pat = pattern_floats(v.n, v.L, pg);
+    p.w_in_smem = (((size_t)v.wsm + pat) * sizeof(float) <= kSmemLimit) ? 1 : 0;
+    size_t need = p.w_in_smem ? (size_t)v.wsm + pat : pat;
+    if (need < (size_t)kGradFloats) need = kGradFloats;
+    p.smem = need * sizeof(float);
     return p;
 }
 

@@ -14,6 +14,9 @@ constexpr int kMaxL = BP_MAX_SIZES - 1;   // weight layers
 constexpr int kFlagTimeout = 1;     // a bounded wait ran out
 constexpr int kFlagNonfinite = 2;   // an error sum was NaN/Inf
 
+// Words of the grid-barrier state (two used, padded to 16 bytes).
+constexpr int kBarWords = 4;
+
 // Device view of a float32 net, passed to kernels by value.
 //   theta/V/G: flat parameter vectors (layer order, W_l row-major then b_l),
 //              P values; wsm = P rounded up to 4 (its shared-memory copy).
@@ -44,7 +47,7 @@ struct F32View {
     float* A;
     float* D;
     float* sse_part;      // one partial error sum per CTA of the pattern phase
-    unsigned* bar;        // grid barrier: [0] arrivals, [1] generation
+    unsigned* bar;        // grid barrier: [0] count at the end of the last launch, [1] arrival count
     int* flags;           // latched error bits
     float lr, momentum, grad_scale;
 };

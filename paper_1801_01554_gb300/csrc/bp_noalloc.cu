@@ -102,10 +102,11 @@ extern "C" bp_status bp_train_epoch_noalloc(const int* layer_sizes, int n_layers
     if (st != BP_OK) return st;
 
     // scratch layout (floats, each part 16-byte aligned):
-    // [error word, pad][barrier x2, pad][per-CTA error sums][activation rows][delta rows]
+    // [error word, pad][barrier words][per-CTA error sums, padded][activation rows][delta rows]
     F32View v{};
     const long long soff = f32_layout(v, layer_sizes, L, minibatch);
-    const long long head = 4 + 4 + (((long long)sms + 3) & ~3LL);
+    const long long bar_words = kBarWords;
+    const long long head = 4 + bar_words + (((long long)sms + 3) & ~3LL);
     const long long need = head + soff;
     if (need > (long long)kNoallocScratchFloats) {
         snprintf(msg, sizeof msg,
@@ -117,7 +118,7 @@ extern "C" bp_status bp_train_epoch_noalloc(const int* layer_sizes, int n_layers
     }
     v.flags = reinterpret_cast<int*>(base);
     v.bar = reinterpret_cast<unsigned*>(base + 4);
-    v.sse_part = base + 8;
+    v.sse_part = base + 4 + bar_words;
     v.A = base + head;
     v.D = base + head + v.a_floats;
     v.theta = d_theta;
@@ -130,7 +131,7 @@ extern "C" bp_status bp_train_epoch_noalloc(const int* layer_sizes, int n_layers
     cudaStream_t s = (cudaStream_t)stream;
     // the array keeps the last call's contents: the error word and the barrier
     // must start at zero
-    cudaError_t e = cudaMemsetAsync(base, 0, 8 * sizeof(float), s);
+    cudaError_t e = cudaMemsetAsync(base, 0, (size_t)(4 + bar_words) * sizeof(float), s);
     if (e == cudaSuccess) {
         const F32Plan plan = f32_plan(v, minibatch, sms);
         const int n_steps = (int)(((long long)n_patterns + minibatch - 1) / minibatch);
