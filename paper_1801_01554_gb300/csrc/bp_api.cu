@@ -197,6 +197,8 @@ bp_status bp_create(const int* sizes, int n_layers, float lr, float momentum, in
         v.G = net->G;
         v.A = net->A;
         v.D = net->D;
+        e = f32_maps(v);
+        if (e != cudaSuccess) return bail(cuda_fail(e, "cuTensorMapEncodeTiled(scratch)"));
         v.sse_part = net->sse_part;
         v.bar = net->bar;
         v.flags = net->flags;
@@ -423,4 +425,18 @@ bp_status bp_train_epoch_host(bp_net* net, const void* h_X, const void* h_T, int
 namespace bp {
 // Lets other translation units report a message through bp_last_error().
 void set_error_message(const char* msg) { g_err = msg; }
+
+PFN_cuTensorMapEncodeTiled_v12000 tensor_map_encoder() {
+    static std::once_flag once;
+    static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+    std::call_once(once, [] {
+        cudaDriverEntryPointQueryResult q;
+        void* p = nullptr;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault,
+                                             &q) == cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
+    });
+    return fn;
+}
 }  // namespace bp

@@ -746,15 +746,8 @@ std::string g_msg;
 PFN_cuTensorMapEncodeTiled_v12000 g_encode = nullptr;
 
 bool get_encoder() {
-    if (g_encode) return true;
-    cudaDriverEntryPointQueryResult q;
-    void* fn = nullptr;
-    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault,
-                                         &q) != cudaSuccess ||
-        q != cudaDriverEntryPointSuccess || fn == nullptr)
-        return false;
-    g_encode = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(fn);
-    return true;
+    if (!g_encode) g_encode = tensor_map_encoder();
+    return g_encode != nullptr;
 }
 
 // 2-D bf16 tensor map over a row-major [rows, cols] matrix with row pitch `ld`

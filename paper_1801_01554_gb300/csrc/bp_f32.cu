@@ -40,7 +40,8 @@ constexpr int kTJ = 32;           // weight-tile columns (inputs; the bias is th
 constexpr int kPC = 256;          // patterns per staged chunk of the weight phase
 constexpr int kPS = kThreads / (kTJ * kTU / 4);   // pattern splits per tile (8)
 constexpr int kChunkFloats = kPC * (kTU + kTJ);
-constexpr size_t kGradFloats = 2 * kChunkFloats + kPS * kTU * kTJ;
+constexpr int kNBuf = 3;          // chunk buffers in flight
+constexpr size_t kGradFloats = kNBuf * kChunkFloats + kPS * kTU * kTJ;
 
 constexpr unsigned long long kWaitNs = 2000000000ull;   // 2 s per wait
 constexpr unsigned kWaitIters = 1u << 26;
@@ -139,6 +140,27 @@ __device__ __forceinline__ void mbar_init1(uint64_t* bar) {
     __syncthreads();
 }
 
+// Waits (bounded) for the phase with the given parity of an mbarrier; on a
+// timeout latches kFlagTimeout and returns false.
+__device__ __forceinline__ bool mbar_wait(uint64_t* bar, unsigned parity, int* flags) {
+    unsigned done = 0;
+    const unsigned long long t0 = global_ns();
+    for (unsigned it = 0;; ++it) {
+        asm volatile(
+            "{\n\t.reg .pred p;\n\t"
+            "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+            "selp.u32 %0, 1, 0, p;\n\t}"
+            : "=r"(done)
+            : "r"(smem_u32(bar)), "r"(parity)
+            : "memory");
+        if (done) return true;
+        if ((it & 255u) == 255u && global_ns() - t0 > kWaitNs) {
+            atomicOr(flags, kFlagTimeout);
+            return false;
+        }
+    }
+}
+
 // Copies theta[0, P) into shared memory Ws (one bulk copy for the 16-byte
 // aligned part, plain loads for the tail).  Bounded wait on the mbarrier.
 __device__ void stage_weights(const float* theta, long long P, float* Ws, uint64_t* bar,
@@ -159,31 +181,13 @@ __device__ void stage_weights(const float* theta, long long P, float* Ws, uint64
     }
     for (long long k = P16 + threadIdx.x; k < P; k += kThreads) Ws[k] = __ldcg(theta + k);
     if (P16 > 0) {
-        unsigned done = 0;
-        const unsigned long long t0 = global_ns();
-        for (unsigned it = 0;; ++it) {
-            asm volatile(
-                "{\n\t.reg .pred p;\n\t"
-                "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
-                "selp.u32 %0, 1, 0, p;\n\t}"
-                : "=r"(done)
-                : "r"(smem_u32(bar)), "r"(phase)
-                : "memory");
-            if (done) break;
-            if ((it & 255u) == 255u && global_ns() - t0 > kWaitNs) {
-                if (threadIdx.x == 0) atomicOr(flags, kFlagTimeout);
-                break;
-            }
-        }
+        mbar_wait(bar, phase, flags);
         phase ^= 1u;
     }
     __syncthreads();
 }
 
 // ------------------------------------------------------------ pattern phase
-__device__ __forceinline__ void cp_async16(float* dst, const float* src) {
-    asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(smem_u32(dst)), "l"(src) : "memory");
-}
 __device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
 template <int N>
 __device__ __forceinline__ void cp_async_wait() { asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory"); }
@@ -376,48 +380,57 @@ __device__ float pattern_phase(const F32View& v, const float* Wb, const float* _
         }
         __syncthreads();
     }
+    // the weight phase reads the activation and delta rows through TMA
+    asm volatile("fence.proxy.async.global;" ::: "memory");
     return block_sum(sse);
 }
 
 // ------------------------------------------------------------ weight phase
 
-// Stage patterns [p0, p0 + pc) of a tile: Ds[pp][0..8) = delta columns u0..,
-// As[pp][0..32) = activation columns j0.. (rows are 16-byte aligned; zeros past
-// the ends of a row and past pc).
-__device__ void stage_tile(float* Ds, float* As, const float* Dl, int dpitch, int u0,
-                           const float* Al, int apitch, int j0, int p0, int pc) {
-    for (int e = threadIdx.x; e < kPC * 10; e += kThreads) {
-        const int pp = e / 10, q = e - pp * 10;
-        float* dst;
-        const float* src;
-        bool ok;
-        if (q < 2) {
-            dst = Ds + pp * kTU + q * 4;
-            ok = pp < pc && u0 + q * 4 < dpitch;
-            src = Dl + (size_t)(p0 + pp) * dpitch + u0 + q * 4;
-        } else {
-            const int c = (q - 2) * 4;
-            dst = As + pp * kTJ + c;
-            ok = pp < pc && j0 + c < apitch;
-            src = Al + (size_t)(p0 + pp) * apitch + j0 + c;
-        }
-        if (ok) {
-            cp_async16(dst, src);
-        } else {
-            *reinterpret_cast<float4*>(dst) = make_float4(0.f, 0.f, 0.f, 0.f);
-        }
-    }
+__device__ __forceinline__ void tma_load_2d(float* smem_dst, const CUtensorMap* map, int c0, int c1,
+                                            uint64_t* bar) {
+    asm volatile(
+        "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes "
+        "[%0], [%1, {%2, %3}], [%4];" ::"r"(smem_u32(smem_dst)),
+        "l"((unsigned long long)map), "r"(c0), "r"(c1), "r"(smem_u32(bar))
+        : "memory");
+}
+
+// Weight-phase pipeline state of a CTA: kNBuf chunk buffers, each filled by two
+// TMA loads that complete on its own mbarrier; `parity` holds one phase bit per
+// buffer and persists across tiles and groups.
+struct ChunkPipe {
+    uint64_t* bar;
+    unsigned parity;
+};
+
+// Issues chunk c of a tile (patterns [c * kPC, c * kPC + kPC)) into buffer
+// c % kNBuf: the [kPC][kTU] delta block at columns u0 of layer l and the
+// [kPC][kTJ] activation block at columns j0 of layer l - 1.  Thread 0 only.
+// Rows and columns past the ends arrive as zeros.
+__device__ __forceinline__ void issue_chunk(const F32View& v, ChunkPipe& pipe, float* smem, int l,
+                                            int u0, int j0, int c) {
+    const int b = c % kNBuf;
+    float* buf = smem + b * kChunkFloats;
+    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_u32(pipe.bar + b)),
+                 "r"((unsigned)(kChunkFloats * sizeof(float)))
+                 : "memory");
+    tma_load_2d(buf, &v.tm_d[l], u0, c * kPC, pipe.bar + b);
+    tma_load_2d(buf + kPC * kTU, &v.tm_a[l - 1], j0, c * kPC, pipe.bar + b);
 }
 
 // Pooled change of every weight (and bias: the last input column is the true
 // unit's 1) over the B patterns of the group, then either accumulate into G
-// (fused == false) or apply the update directly.
-__device__ void weight_phase(const F32View& v, int B, bool fused, bool fold_g, float* smem) {
+// (fused == false) or apply the update directly.  One CTA per 8 x 32 tile;
+// the tile's delta and activation columns stream through shared memory in
+// chunks of kPC patterns by TMA, kNBuf chunks in flight.
+__device__ void weight_phase(const F32View& v, int B, bool fused, bool fold_g, float* smem,
+                             ChunkPipe& pipe) {
     const int tid = threadIdx.x;
     // thread = (pattern split ps, 4 output units uq, input column j)
     const int ps = tid / (kTJ * kTU / 4), r = tid - ps * (kTJ * kTU / 4);
     const int uq = r / kTJ, j = r - uq * kTJ;
-    float* red = smem + 2 * kChunkFloats;   // [kPS][kTU][kTJ]
+    float* red = smem + kNBuf * kChunkFloats;   // [kPS][kTU][kTJ]
     const int L = v.L;
     const int ntiles = v.tile0[L + 1];
     const int nchunks = (B + kPC - 1) / kPC;
@@ -429,26 +442,28 @@ __device__ void weight_phase(const F32View& v, int B, bool fused, bool fold_g, f
         const int tb = lt / v.tcols[l], cb = lt - tb * v.tcols[l];
         const int n_in = v.n[l - 1], n_out = v.n[l];
         const int u0 = tb * kTU, j0 = cb * kTJ;
-        const float* Dl = v.D + v.doff[l];
-        const float* Al = v.A + v.aoff[l - 1];
         float acc[4] = {0.f, 0.f, 0.f, 0.f};
-        stage_tile(smem, smem + kPC * kTU, Dl, v.dpitch[l], u0, Al, v.apitch[l - 1], j0, 0,
-                   min(kPC, B));
-        cp_async_commit();
+        // the buffers' previous contents (weights, pattern rows, the last tile)
+        // were read through the generic proxy by every thread before this sync
+        __syncthreads();
+        if (tid == 0) {
+            asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+            asm volatile("fence.proxy.async.global;" ::: "memory");
+            for (int c = 0; c < nchunks && c < kNBuf; ++c) issue_chunk(v, pipe, smem, l, u0, j0, c);
+        }
         for (int c = 0; c < nchunks; ++c) {
-            if (c + 1 < nchunks) {
-                const int p0 = (c + 1) * kPC;
-                float* nb = smem + ((c + 1) & 1) * kChunkFloats;
-                stage_tile(nb, nb + kPC * kTU, Dl, v.dpitch[l], u0, Al, v.apitch[l - 1], j0, p0,
-                           min(kPC, B - p0));
-                cp_async_commit();
-                cp_async_wait<1>();
-            } else {
-                cp_async_wait<0>();
+            const int b = c % kNBuf;
+            mbar_wait(pipe.bar + b, (pipe.parity >> b) & 1u, v.flags);
+            pipe.parity ^= 1u << b;
+            float* Ds = smem + b * kChunkFloats;
+            float* As = Ds + kPC * kTU;
+            const int pc = B - c * kPC;
+            if (pc < kPC) {
+                // rows past the group may hold stale scratch rows: clear them
+                for (int e = tid; e < (kPC - pc) * kTU; e += kThreads) Ds[pc * kTU + e] = 0.f;
+                for (int e = tid; e < (kPC - pc) * kTJ; e += kThreads) As[pc * kTJ + e] = 0.f;
+                __syncthreads();
             }
-            __syncthreads();
-            const float* Ds = smem + (c & 1) * kChunkFloats;
-            const float* As = Ds + kPC * kTU;
             const int pp0 = ps * kPer;
 #pragma unroll 4
             for (int k = 0; k < kPer; ++k) {
@@ -461,6 +476,10 @@ __device__ void weight_phase(const F32View& v, int B, bool fused, bool fold_g, f
                 acc[3] = fmaf(d.w, a, acc[3]);
             }
             __syncthreads();
+            if (tid == 0 && c + kNBuf < nchunks) {
+                asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+                issue_chunk(v, pipe, smem, l, u0, j0, c + kNBuf);
+            }
         }
 #pragma unroll
         for (int k = 0; k < 4; ++k) red[(ps * kTU + uq * 4 + k) * kTJ + j] = acc[k];
@@ -485,9 +504,22 @@ __device__ void weight_phase(const F32View& v, int B, bool fused, bool fold_g, f
                     v.theta[idx] += vel;
                 }
             }
+            // the next group's bulk copy reads theta through the async proxy
+            asm volatile("fence.proxy.async.global;" ::: "memory");
         }
-        __syncthreads();
     }
+}
+
+// Initialises the weight-phase mbarriers (static shared memory) of a launch.
+__device__ void pipe_init(ChunkPipe& pipe, uint64_t* bars) {
+    if (threadIdx.x == 0) {
+        for (int b = 0; b < kNBuf; ++b)
+            asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(smem_u32(bars + b)) : "memory");
+        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    }
+    __syncthreads();
+    pipe.bar = bars;
+    pipe.parity = 0;
 }
 
 // Error sum of the group by the first warp of the last CTA: lane-strided
@@ -507,8 +539,9 @@ __device__ void reduce_sse(const F32View& v, int nparts, float* sse_out) {
 // ------------------------------------------------------------ kernels
 // WS: the weights are copied into shared memory (else read from global memory).
 template <int PG, bool WS>
-__global__ void __launch_bounds__(kThreads, 1) k_forward(F32View v, const float* X, int B, float* Y) {
-    extern __shared__ __align__(16) float smem[];
+__global__ void __launch_bounds__(kThreads, 1)
+    k_forward(const __grid_constant__ F32View v, const float* X, int B, float* Y) {
+    extern __shared__ __align__(128) float smem[];
     __shared__ __align__(8) uint64_t s_bar;
     unsigned phase = 0;
     if (WS) {
@@ -521,8 +554,9 @@ __global__ void __launch_bounds__(kThreads, 1) k_forward(F32View v, const float*
 }
 
 template <int PG, bool WS>
-__global__ void __launch_bounds__(kThreads, 1) k_deltas(F32View v, const float* T, int B) {
-    extern __shared__ __align__(16) float smem[];
+__global__ void __launch_bounds__(kThreads, 1)
+    k_deltas(const __grid_constant__ F32View v, const float* T, int B) {
+    extern __shared__ __align__(128) float smem[];
     __shared__ __align__(8) uint64_t s_bar;
     unsigned phase = 0;
     float e;
@@ -537,13 +571,16 @@ __global__ void __launch_bounds__(kThreads, 1) k_deltas(F32View v, const float* 
 }
 
 __global__ void __launch_bounds__(kThreads, 1)
-    k_accumulate(F32View v, int B, int nparts, float* sse_out) {
-    extern __shared__ __align__(16) float smem[];
+    k_accumulate(const __grid_constant__ F32View v, int B, int nparts, float* sse_out) {
+    extern __shared__ __align__(128) float smem[];
+    __shared__ __align__(8) uint64_t s_cbar[kNBuf];
+    ChunkPipe pipe;
+    pipe_init(pipe, s_cbar);
     reduce_sse(v, nparts, sse_out);
-    weight_phase(v, B, false, false, smem);
+    weight_phase(v, B, false, false, smem, pipe);
 }
 
-__global__ void __launch_bounds__(256) k_update(F32View v, long long n) {
+__global__ void __launch_bounds__(256) k_update(const __grid_constant__ F32View v, long long n) {
     const float a = v.lr * v.grad_scale, m = v.momentum;
     for (long long k = blockIdx.x * 256LL + threadIdx.x; k < n; k += (long long)gridDim.x * 256) {
         const float vel = a * v.G[k] + m * v.V[k];
@@ -555,15 +592,18 @@ __global__ void __launch_bounds__(256) k_update(F32View v, long long n) {
 
 template <int PG, bool WS>
 __global__ void __launch_bounds__(kThreads, 1)
-    k_train(F32View v, const float* X, const float* T, int n_patterns, int minibatch, int n_steps,
-            float* sse_out, int fold_g) {
-    extern __shared__ __align__(16) float smem[];
+    k_train(const __grid_constant__ F32View v, const float* X, const float* T, int n_patterns,
+            int minibatch, int n_steps, float* sse_out, int fold_g) {
+    extern __shared__ __align__(128) float smem[];
     __shared__ __align__(8) uint64_t s_bar;
+    __shared__ __align__(8) uint64_t s_cbar[kNBuf];
     // A latched timeout means an earlier launch left the barrier half-way; do
     // nothing until bp_check() has cleared the latch and reset the barrier.
     if (__ldcg(v.flags) & kFlagTimeout) return;
     unsigned phase = 0;
     mbar_init1(&s_bar);
+    ChunkPipe pipe;
+    pipe_init(pipe, s_cbar);
     // arrival count at the end of the previous launch; barrier k waits for
     // base + k * grid arrivals
     unsigned target = __ldcg(v.bar);
@@ -584,7 +624,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (threadIdx.x == 0) v.sse_part[blockIdx.x] = e;
         if (!grid_barrier(v.bar, target += gridDim.x, v.flags)) return;
         reduce_sse(v, gridDim.x, sse_out != nullptr ? sse_out + s : nullptr);
-        weight_phase(v, B, true, fold_g != 0 && s == 0, smem);
+        weight_phase(v, B, true, fold_g != 0 && s == 0, smem, pipe);
         if (s + 1 < n_steps) {
             if (!grid_barrier(v.bar, target += gridDim.x, v.flags)) return;
         }
@@ -675,6 +715,29 @@ int f32_max_pg(const int* n, int L) {
     for (int pg = 1; pg <= 8; pg *= 2)
         if (f32_smem_bytes(n, L, pg) <= kSmemLimit) best = pg;
     return best;
+}
+
+// One float32 2-D map over rows [rows][pitch] (pitch floats apart), boxes of
+// box_cols x kPC, zero fill outside.
+static bool encode_rows(CUtensorMap* map, const float* base, int rows, int pitch, int box_cols) {
+    PFN_cuTensorMapEncodeTiled_v12000 enc = tensor_map_encoder();
+    if (enc == nullptr) return false;
+    cuuint64_t dims[2] = {(cuuint64_t)pitch, (cuuint64_t)rows};
+    cuuint64_t strides[1] = {(cuuint64_t)pitch * sizeof(float)};
+    cuuint32_t box[2] = {(cuuint32_t)box_cols, (cuuint32_t)kPC};
+    cuuint32_t estr[2] = {1, 1};
+    return enc(map, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 2, const_cast<float*>(base), dims, strides, box,
+               estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE,
+               CU_TENSOR_MAP_L2_PROMOTION_L2_128B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+cudaError_t f32_maps(F32View& v) {
+    for (int l = 1; l <= v.L; ++l) {
+        if (!encode_rows(&v.tm_d[l], v.D + v.doff[l], v.cap, v.dpitch[l], kTU) ||
+            !encode_rows(&v.tm_a[l - 1], v.A + v.aoff[l - 1], v.cap, v.apitch[l - 1], kTJ))
+            return cudaErrorInvalidValue;
+    }
+    return cudaSuccess;
 }
 
 cudaError_t f32_setup(int device) {

@@ -1,7 +1,9 @@
 // Internal declarations shared by the translation units of libbp.so.
 #pragma once
 
+#include <cuda.h>
 #include <cuda_runtime.h>
+#include <cudaTypedefs.h>
 #include <cstdint>
 
 #include "bp.h"
@@ -50,6 +52,13 @@ struct F32View {
     unsigned* bar;        // grid barrier: [0] count at the end of the last launch, [1] arrival count
     int* flags;           // latched error bits
     float lr, momentum, grad_scale;
+    // TMA maps of the weight phase (f32_maps): tm_d[l] over the delta rows of
+    // layer l (boxes of 8 columns x 256 patterns), tm_a[l] over the activation
+    // rows of layer l (boxes of 32 columns x 256 patterns); zero fill past the
+    // row pitch and past `cap`.  Kernels take the view as a __grid_constant__
+    // parameter so that the maps can be addressed in place.
+    CUtensorMap tm_d[BP_MAX_SIZES];
+    CUtensorMap tm_a[BP_MAX_SIZES];
 };
 
 // Launch geometry chosen on the host for a group size.
@@ -68,6 +77,8 @@ long long f32_layout(F32View& v, const int* n, int L, int cap);
 int f32_max_pg(const int* n, int L);
 size_t f32_smem_bytes(const int* n, int L, int pg);
 cudaError_t f32_setup(int device);   // opt-in shared memory limits, once per process
+// Encodes the TMA maps of v over its A and D buffers (set A, D and the layout first).
+cudaError_t f32_maps(F32View& v);
 F32Plan f32_plan(const F32View& v, int batch, int num_sms);
 
 cudaError_t f32_forward(const F32View& v, const float* X, int batch, float* Y,
@@ -84,5 +95,9 @@ cudaError_t f32_train(const F32View& v, const float* X, const float* T, int n_pa
 
 // Message returned by bp_last_error() on the calling thread (bp_api.cu).
 void set_error_message(const char* msg);
+
+// cuTensorMapEncodeTiled from the driver, looked up once (bp_api.cu); null if
+// the driver does not provide it.
+PFN_cuTensorMapEncodeTiled_v12000 tensor_map_encoder();
 
 }  // namespace bp

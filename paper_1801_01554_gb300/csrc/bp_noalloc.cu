@@ -121,6 +121,10 @@ extern "C" bp_status bp_train_epoch_noalloc(const int* layer_sizes, int n_layers
     v.sse_part = base + 4 + bar_words;
     v.A = base + head;
     v.D = base + head + v.a_floats;
+    if (f32_maps(v) != cudaSuccess) {
+        set_error_message("bp_train_epoch_noalloc: cuTensorMapEncodeTiled failed for the scratch");
+        return BP_ECUDA;
+    }
     v.theta = d_theta;
     v.V = d_V;
     v.G = nullptr;   // nothing pending: the launch never reads G
