@@ -260,7 +260,8 @@ def run_ours(args, world, rank, local):
     # runs in its own interpreter), on rank 0 only, single-GPU runs only.
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        r = time_oracle(n, 60.0, min_s=args.cpu_seconds, max_epochs=w["epochs"],
+        # whole epochs until at least --cpu-seconds of CPU work (60 s cap)
+        r = time_oracle(n, 60.0, min_s=args.cpu_seconds, max_epochs=10 ** 6,
                         workload=args.workload)[0]
         cpu = {"value": W * r["patterns"] / r["seconds"], "unit": UNIT, "cores": 1,
                "kind": "oracle",
