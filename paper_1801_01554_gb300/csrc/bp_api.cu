@@ -8,6 +8,7 @@
 #include <cstring>
 #include <mutex>
 #include <string>
+#include <vector>
 
 #include "bp.h"
 #include "bp_bf16.h"
@@ -52,7 +53,8 @@ struct bp_net {
     int max_batch = 0;
     int device = 0;
     int num_sms = 0;
-    long long P = 0;
+    long long P = 0;    // parameters in the API's packed layout
+    long long Pd = 0;   // floats of theta, V and G on the device (padded for float32)
     float lr = 0.f, momentum = 0.f, grad_scale = 1.f;
     // float32 master state (both paths)
     float* theta = nullptr;
@@ -140,6 +142,7 @@ bp_status bp_create(const int* sizes, int n_layers, float lr, float momentum, in
     long long P = 0;
     for (int l = 1; l <= net->L; ++l) P += (long long)(sizes[l - 1] + 1) * sizes[l];
     net->P = P;
+    net->Pd = P;
 
     auto bail = [&](bp_status st) {
         free_all(net);
@@ -169,18 +172,23 @@ bp_status bp_create(const int* sizes, int n_layers, float lr, float momentum, in
         if (st != BP_OK) return bail(fail(st, "%s", bf16_last_message()));
     }
 
-    e = cudaMalloc(&net->theta, P * sizeof(float));
-    if (e == cudaSuccess) e = cudaMalloc(&net->V, P * sizeof(float));
-    if (e == cudaSuccess) e = cudaMalloc(&net->G, P * sizeof(float));
+    // float32 nets keep their parameters in the padded device layout
+    if (dtype == BP_F32) {
+        f32_layout(net->view, net->n, net->L, max_batch);
+        net->Pd = net->view.P;
+    }
+    const long long Pd = net->Pd;
+    e = cudaMalloc(&net->theta, Pd * sizeof(float));
+    if (e == cudaSuccess) e = cudaMalloc(&net->V, Pd * sizeof(float));
+    if (e == cudaSuccess) e = cudaMalloc(&net->G, Pd * sizeof(float));
     if (e != cudaSuccess) return bail(cuda_fail(e, "cudaMalloc(parameters)"));
-    e = cudaMemset(net->theta, 0, P * sizeof(float));
-    if (e == cudaSuccess) e = cudaMemset(net->V, 0, P * sizeof(float));
-    if (e == cudaSuccess) e = cudaMemset(net->G, 0, P * sizeof(float));
+    e = cudaMemset(net->theta, 0, Pd * sizeof(float));
+    if (e == cudaSuccess) e = cudaMemset(net->V, 0, Pd * sizeof(float));
+    if (e == cudaSuccess) e = cudaMemset(net->G, 0, Pd * sizeof(float));
     if (e != cudaSuccess) return bail(cuda_fail(e, "cudaMemset(parameters)"));
 
     if (dtype == BP_F32) {
         F32View& v = net->view;
-        f32_layout(v, net->n, net->L, max_batch);
         e = cudaMalloc(&net->A, v.a_floats * sizeof(float));
         if (e == cudaSuccess) e = cudaMalloc(&net->D, v.d_floats * sizeof(float));
         if (e == cudaSuccess) e = cudaMalloc(&net->sse_part, (size_t)net->num_sms * 4 * sizeof(float));
@@ -238,13 +246,26 @@ bp_status bp_set_hparams(bp_net* net, float lr, float momentum, float grad_scale
 
 int64_t bp_num_params(const bp_net* net) { return net ? (int64_t)net->P : 0; }
 
+// Copies a parameter vector between the caller's packed layout (host) and the
+// net's device layout (padded for float32 nets).
 static bp_status copy_params(const bp_net* net, float* dst, const float* src, bool to_device,
                              const char* what) {
     if (net == nullptr || dst == nullptr || src == nullptr) return fail(BP_EINVAL, "NULL argument");
     BP_CUDA(cudaDeviceSynchronize(), what);
-    BP_CUDA(cudaMemcpy(dst, src, net->P * sizeof(float),
-                       to_device ? cudaMemcpyHostToDevice : cudaMemcpyDeviceToHost),
-            what);
+    if (net->dtype != BP_F32) {
+        BP_CUDA(cudaMemcpy(dst, src, net->P * sizeof(float),
+                           to_device ? cudaMemcpyHostToDevice : cudaMemcpyDeviceToHost),
+                what);
+        return BP_OK;
+    }
+    std::vector<float> tmp((size_t)net->Pd);
+    if (to_device) {
+        f32_pad_host(net->view, src, tmp.data());
+        BP_CUDA(cudaMemcpy(dst, tmp.data(), net->Pd * sizeof(float), cudaMemcpyHostToDevice), what);
+    } else {
+        BP_CUDA(cudaMemcpy(tmp.data(), src, net->Pd * sizeof(float), cudaMemcpyDeviceToHost), what);
+        f32_unpad_host(net->view, tmp.data(), dst);
+    }
     return BP_OK;
 }
 
@@ -318,7 +339,7 @@ bp_status bp_update(bp_net* net, void* stream) {
     if (net == nullptr) return fail(BP_EINVAL, "NULL net");
     cudaStream_t s = (cudaStream_t)stream;
     if (net->dtype == BP_F32) {
-        BP_CUDA(f32_update(net->view, net->P, s), "bp_update");
+        BP_CUDA(f32_update(net->view, net->Pd, s), "bp_update");
     } else {
         BP_CUDA(bf16_update(net->bf, net->lr, net->momentum, net->grad_scale, s), "bp_update");
     }

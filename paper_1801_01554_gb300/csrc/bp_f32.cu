@@ -115,22 +115,6 @@ __device__ float block_sum(float x) {
     return r;
 }
 
-// Butterfly reduce-scatter of 32 per-lane values: afterwards lane k holds in
-// v[0] the warp-wide sum of value k.  A binary-tree sum of each dot product
-// (Section 10.3), 31 shuffles for 32 sums.
-__device__ __forceinline__ void reduce_scatter32(float (&v)[32], int lane) {
-#pragma unroll
-    for (int half = 16; half >= 1; half >>= 1) {
-        const bool up = (lane & half) != 0;
-#pragma unroll
-        for (int k = 0; k < half; ++k) {
-            const float send = up ? v[k] : v[k + half];
-            const float keep = up ? v[k + half] : v[k];
-            v[k] = keep + __shfl_xor_sync(0xffffffffu, send, half);
-        }
-    }
-}
-
 // ------------------------------------------------------------ weights in shared memory
 __device__ __forceinline__ void mbar_init1(uint64_t* bar) {
     if (threadIdx.x == 0) {
@@ -202,181 +186,315 @@ __device__ __forceinline__ float* pattern_base(const F32View& v, float* smem) {
     return WS ? smem + v.wsm : smem;
 }
 
-// Offset of the target rows inside the pattern buffers (after the activation
-// and delta rows of PG patterns).
-template <int PG>
-__device__ __forceinline__ int target_offset(const F32View& v) {
-    int units = 0;
-    for (int l = 0; l <= v.L; ++l) units += v.n[l];
-    for (int l = 1; l <= v.L; ++l) units += v.n[l];
-    return PG * units;
-}
+// Pattern buffers (PatLayout, computed on the host): the activation rows keep
+// the true unit's 1 in column n_l and zeros after it, so that a padded weight
+// row times an activation row is the unit's net input with its bias.
+//
+// Row loops below give each pattern kThreads / PG threads (a compile-time
+// split: pattern = thread / TP, column = thread % TP), so no thread divides.
 
-// Issues the copies of the input rows (into sx, [PG][n0]) and target rows (into
-// st, [PG][nL]) of patterns [p0, p0 + np); rows past np are zeroed.  One
-// cp.async group; the caller waits for it before use.  (Issuing them one group
-// ahead, to land during the barrier and the weight phase, measured no faster.)
+// Issues the copies of the input rows (into the layer-0 activation rows) and
+// target rows of patterns [p0, p0 + np), and writes the true unit's 1 and the
+// zero pads of every activation and delta row; rows past np are zeroed.  One
+// cp.async group; the caller waits for it before use.
 template <int PG>
-__device__ void load_rows(const float* X, const float* T, int n0, int nL, int p0, int np, float* sx,
-                          float* st) {
+__device__ void load_rows(const F32View& v, const PatLayout& q, const float* X, const float* T,
+                          int p0, int np, float* smem) {
+    constexpr int TP = kThreads / PG;
+    const int p = threadIdx.x / TP, c0 = threadIdx.x % TP;
+    const bool live = p < np;
+    const int n0 = v.n[0], nL = v.n[v.L];
     if (X != nullptr) {
-        for (int e = threadIdx.x; e < PG * n0; e += kThreads) {
-            const int p = e / n0, i = e - p * n0;
-            if (p < np) cp_async4(sx + e, X + (size_t)(p0 + p) * n0 + i);
-            else sx[e] = 0.f;
+        float* dst = smem + q.sa[0] + p * v.apitch[0];
+        const float* src = X + (size_t)(p0 + p) * n0;
+        for (int i = c0; i < n0; i += TP) {
+            if (live) cp_async4(dst + i, src + i);
+            else dst[i] = 0.f;
         }
     }
     if (T != nullptr) {
-        for (int e = threadIdx.x; e < PG * nL; e += kThreads) {
-            const int p = e / nL, k = e - p * nL;
-            if (p < np) cp_async4(st + e, T + (size_t)(p0 + p) * nL + k);
-            else st[e] = 0.f;
+        float* dst = smem + q.st + p * nL;
+        const float* src = T + (size_t)(p0 + p) * nL;
+        for (int k = c0; k < nL; k += TP) {
+            if (live) cp_async4(dst + k, src + k);
+            else dst[k] = 0.f;
         }
     }
     cp_async_commit();
+    // pads: at most 4 columns per row (apitch - n in [1, 4], dpitch - n in [0, 3])
+    if (c0 < 4) {
+        for (int l = 0; l <= v.L; ++l) {
+            const int col = v.n[l] + c0;
+            if (col < v.apitch[l]) smem[q.sa[l] + p * v.apitch[l] + col] = (c0 == 0) ? 1.f : 0.f;
+            if (l >= 1 && col < v.dpitch[l]) smem[q.sd[l] + p * v.dpitch[l] + col] = 0.f;
+        }
+    }
 }
 
-// Forward through one layer for PG patterns held in shared memory:
-// out[p][j] = sigma(sum_i W[j][i] in[p][i] + b[j]).  A warp owns 32/PG units at
-// a time; lanes stride over the inputs.
+// Butterfly reduce-scatter of V per-lane values over aligned groups of V lanes:
+// afterwards lane k of a group holds in v[0] the group's sum of value k mod V.
+// A binary-tree sum (Section 10.3), V - 1 shuffles for V sums.
+template <int V>
+__device__ __forceinline__ void reduce_scatter(float (&v)[V], int lane) {
+#pragma unroll
+    for (int half = V / 2; half >= 1; half >>= 1) {
+        const bool up = (lane & half) != 0;
+#pragma unroll
+        for (int k = 0; k < half; ++k) {
+            const float send = up ? v[k] : v[k + half];
+            const float keep = up ? v[k + half] : v[k];
+            v[k] = keep + __shfl_xor_sync(0xffffffffu, send, half);
+        }
+    }
+}
+
+__device__ __forceinline__ float4 ld4(const float* p) { return *reinterpret_cast<const float4*>(p); }
+
+// Units per lane group of the forward pass for a group size: every unit's
+// weights are read once per CTA, every activation row once per lane group.
 template <int PG>
-__device__ void forward_layer(const float* W, const float* b, int n_in, int n_out, const float* s_in,
-                              float* s_out) {
-    constexpr int UJ = 32 / PG;
-    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-    for (int j0 = warp * UJ; j0 < n_out; j0 += kWarps * UJ) {
-        float acc[32];
+constexpr int fwd_units() { return PG >= 8 ? 4 : 8 / PG; }
+
+// Forward through one layer for PG patterns held in shared memory:
+// out[p][j] = sigma(sum_i W[j][i] in[p][i]) over the kp columns of the padded
+// rows (the bias column meets the activation row's 1).  A group of S lanes
+// (V = U * PG, 2V or 4V up to 32; within one warp) owns U units and sums V
+// dot products over interleaved float4 columns, then reduces them across its
+// lanes: a reduce-scatter inside each V-lane block, then butterflies across
+// blocks.
+template <int PG>
+__device__ void forward_layer(const float* W, int kp, int n_out, const float* s_in, float* s_out,
+                              int kp_out) {
+    constexpr int U = fwd_units<PG>();
+    constexpr int V = U * PG;
+    static_assert(V <= 32, "a lane group holds at most 32 sums");
+    const int G = (n_out + U - 1) / U;
+    int S = 32;
+    while (S > V && G * S > kThreads) S >>= 1;
+    const int gpp = kThreads / S;
+    const int tid = threadIdx.x, lane = tid & 31;
+    const int s = tid & (S - 1), g0 = tid / S;
+    const int K4 = kp >> 2;
+    for (int gb = 0; gb < G; gb += gpp) {   // uniform trip count: every lane shuffles
+        const int g = gb + g0;
+        const int j0 = g * U;
+        float acc[V];
 #pragma unroll
-        for (int k = 0; k < 32; ++k) acc[k] = 0.f;
-        for (int i = lane; i < n_in; i += 32) {
-            float a[PG];
+        for (int k = 0; k < V; ++k) acc[k] = 0.f;
+        if (g < G) {
+            const float* wr[U];
 #pragma unroll
-            for (int p = 0; p < PG; ++p) a[p] = s_in[p * n_in + i];
+            for (int u = 0; u < U; ++u) wr[u] = W + (size_t)min(j0 + u, n_out - 1) * kp;
+            for (int k = s; k < K4; k += S) {
+                float4 a[PG];
 #pragma unroll
-            for (int u = 0; u < UJ; ++u) {
-                const int j = min(j0 + u, n_out - 1);   // rows past the end are discarded
-                const float w = W[(size_t)j * n_in + i];
+                for (int p = 0; p < PG; ++p) a[p] = ld4(s_in + p * kp + 4 * k);
 #pragma unroll
-                for (int p = 0; p < PG; ++p) acc[u * PG + p] = fmaf(w, a[p], acc[u * PG + p]);
+                for (int u = 0; u < U; ++u) {
+                    const float4 w = ld4(wr[u] + 4 * k);
+#pragma unroll
+                    for (int p = 0; p < PG; ++p) {
+                        float t = acc[u * PG + p];
+                        t = fmaf(w.x, a[p].x, t);
+                        t = fmaf(w.y, a[p].y, t);
+                        t = fmaf(w.z, a[p].z, t);
+                        t = fmaf(w.w, a[p].w, t);
+                        acc[u * PG + p] = t;
+                    }
+                }
             }
         }
-        reduce_scatter32(acc, lane);
-        const int u = lane / PG, p = lane % PG;
-        const int j = j0 + u;
-        if (j < n_out) s_out[p * n_out + j] = sigmoid_f(acc[0] + b[j]);
+        reduce_scatter<V>(acc, lane);
+        float r = acc[0];
+        for (int o = V; o < S; o <<= 1) r += __shfl_xor_sync(0xffffffffu, r, o);
+        if (s < V && g < G) {
+            const int u = s / PG, p = s % PG;
+            const int j = j0 + u;
+            if (j < n_out) s_out[p * kp_out + j] = sigmoid_f(r);
+        }
+    }
+}
+
+// PG consecutive floats (16-byte aligned when PG >= 4) into registers.
+template <int PG>
+__device__ __forceinline__ void load_pg(const float* p, float (&d)[PG]) {
+    if constexpr (PG >= 4) {
+#pragma unroll
+        for (int k = 0; k < PG; k += 4) {
+            const float4 x = *reinterpret_cast<const float4*>(p + k);
+            d[k] = x.x;
+            d[k + 1] = x.y;
+            d[k + 2] = x.z;
+            d[k + 3] = x.w;
+        }
+    } else if constexpr (PG == 2) {
+        const float2 x = *reinterpret_cast<const float2*>(p);
+        d[0] = x.x;
+        d[1] = x.y;
+    } else {
+        d[0] = p[0];
+    }
+}
+
+// Hidden deltas of layer l for PG patterns: d_l[p][i] = (sum_j W_{l+1}[j][i]
+// d_{l+1}[p][j]) a_l[p][i] (1 - a_l[p][i]).  dnt holds d_{l+1} pattern-minor
+// ([nn][PG]) so that one vector load gives a column's PG deltas.  Units go to
+// threads; when there are fewer than kThreads units, the sum over j is split
+// over JS interleaved slices whose partials meet in shared memory in a fixed
+// order.  Writes d_l as rows (dl, pitch dpl) and, if dlt is not null,
+// pattern-minor (dlt).
+template <int PG>
+__device__ void hidden_delta(const float* Wn, int kpn, int n, int nn, const float* dnt,
+                             const float* al, int apl, float* dl, int dpl, float* dlt, float* red) {
+    const int tid = threadIdx.x;
+    const int NI = (n + 31) & ~31;
+    const int JS = NI < kThreads ? kThreads / NI : 1;
+    if (JS > 1) {
+        const int sl = tid / NI, i = tid - sl * NI;
+        float acc[PG];
+#pragma unroll
+        for (int p = 0; p < PG; ++p) acc[p] = 0.f;
+        if (sl < JS && i < n) {
+#pragma unroll 2
+            for (int j = sl; j < nn; j += JS) {
+                const float w = Wn[(size_t)j * kpn + i];
+                float d[PG];
+                load_pg<PG>(dnt + j * PG, d);
+#pragma unroll
+                for (int p = 0; p < PG; ++p) acc[p] = fmaf(d[p], w, acc[p]);
+            }
+        }
+        if (sl < JS) {
+#pragma unroll
+            for (int p = 0; p < PG; ++p) red[(sl * PG + p) * NI + i] = acc[p];
+        }
+        __syncthreads();
+        if (tid < n) {
+#pragma unroll
+            for (int p = 0; p < PG; ++p) {
+                float g = 0.f;
+                for (int k = 0; k < JS; ++k) g += red[(k * PG + p) * NI + tid];
+                const float a = al[p * apl + tid];
+                const float d = g * a * (1.f - a);
+                dl[p * dpl + tid] = d;
+                if (dlt != nullptr) dlt[tid * PG + p] = d;
+            }
+        }
+    } else {
+        for (int i = tid; i < n; i += kThreads) {
+            float acc[PG];
+#pragma unroll
+            for (int p = 0; p < PG; ++p) acc[p] = 0.f;
+#pragma unroll 2
+            for (int j = 0; j < nn; ++j) {
+                const float w = Wn[(size_t)j * kpn + i];
+                float d[PG];
+                load_pg<PG>(dnt + j * PG, d);
+#pragma unroll
+                for (int p = 0; p < PG; ++p) acc[p] = fmaf(d[p], w, acc[p]);
+            }
+#pragma unroll
+            for (int p = 0; p < PG; ++p) {
+                const float a = al[p * apl + i];
+                const float d = acc[p] * a * (1.f - a);
+                dl[p * dpl + i] = d;
+                if (dlt != nullptr) dlt[i * PG + p] = d;
+            }
+        }
+    }
+}
+
+// Copies np rows of `pitch` floats (a multiple of 4) from shared to global
+// memory as float4.
+template <int PG>
+__device__ __forceinline__ void rows_to_global(float* dst, const float* src, int pitch, int np) {
+    constexpr int TP = kThreads / PG;
+    const int p = threadIdx.x / TP, c0 = threadIdx.x % TP;
+    if (p < np) {
+        const int q4 = pitch >> 2;
+        float4* d = reinterpret_cast<float4*>(dst + (size_t)p * pitch);
+        const float4* s = reinterpret_cast<const float4*>(src + p * pitch);
+        for (int c = c0; c < q4; c += TP) d[c] = s[c];
     }
 }
 
 // Runs the pattern phase for this CTA's share of the group's B patterns
 // (patterns [blockIdx.x*B/gridDim.x, (blockIdx.x+1)*B/gridDim.x), PG at a time).
-//   Wb: the weights (shared memory copy or global theta)
+//   Wb: the weights in the padded layout (shared memory copy or global theta)
+//   q: the pattern buffers' layout, relative to smem
 //   do_fwd: forward pass from X (else the activations are reloaded from scratch)
 //   do_bwd: deltas against T, written to scratch
 //   Y: if not null, the outputs are copied there ([B, n_L] packed)
 // Returns this CTA's summed squared error (valid in thread 0).
 template <int PG>
-__device__ float pattern_phase(const F32View& v, const float* Wb, const float* __restrict__ X,
-                               const float* __restrict__ T, int B, bool do_fwd, bool do_bwd,
-                               float* __restrict__ Y, float* smem) {
+__device__ float pattern_phase(const F32View& v, const PatLayout& q, const float* Wb,
+                               const float* __restrict__ X, const float* __restrict__ T, int B,
+                               bool do_fwd, bool do_bwd, float* __restrict__ Y, float* smem) {
+    constexpr int TP = kThreads / PG;
     const int L = v.L;
     const int tid = threadIdx.x;
-    const int n0 = v.n[0], nL = v.n[L];
-    int sa[BP_MAX_SIZES], sd[BP_MAX_SIZES];
-    {
-        int off = 0;
-        for (int l = 0; l <= L; ++l) { sa[l] = off; off += PG * v.n[l]; }
-        for (int l = 1; l <= L; ++l) { sd[l] = off; off += PG * v.n[l]; }
-    }
-    const int st = target_offset<PG>(v);
+    const int pr = tid / TP, c0 = tid % TP;   // row-loop split
+    const int nL = v.n[L];
     float sse = 0.f;
     const int q_lo = (int)((long long)B * blockIdx.x / gridDim.x);
     const int q_hi = (int)((long long)B * (blockIdx.x + 1) / gridDim.x);
     for (int p0 = q_lo; p0 < q_hi; p0 += PG) {
         const int np = min(PG, q_hi - p0);
-        load_rows<PG>(do_fwd ? X : nullptr, do_bwd ? T : nullptr, n0, nL, p0, np, smem + sa[0],
-                      smem + st);
+        load_rows<PG>(v, q, do_fwd ? X : nullptr, do_bwd ? T : nullptr, p0, np, smem);
+        if (!do_fwd) {
+            // activations of the last forward, reloaded from scratch
+            for (int l = 1; l <= L; ++l) {
+                const int ap = v.apitch[l], q4 = ap >> 2;
+                const float4* src =
+                    reinterpret_cast<const float4*>(v.A + v.aoff[l] + (size_t)(p0 + pr) * ap);
+                float4* dst = reinterpret_cast<float4*>(smem + q.sa[l] + pr * ap);
+                for (int c = c0; c < q4; c += TP)
+                    dst[c] = (pr < np) ? __ldcg(src + c) : make_float4(0.f, 0.f, 0.f, 0.f);
+            }
+        }
         cp_async_wait<0>();
         __syncthreads();
         if (do_fwd) {
             for (int l = 1; l <= L; ++l) {
-                forward_layer<PG>(Wb + v.woff[l], Wb + v.boff[l], v.n[l - 1], v.n[l], smem + sa[l - 1],
-                                  smem + sa[l]);
+                forward_layer<PG>(Wb + v.woff[l], v.kp[l], v.n[l], smem + q.sa[l - 1], smem + q.sa[l],
+                                  v.apitch[l]);
                 __syncthreads();
             }
-            // activation rows (a trailing 1 is the true unit's input, zeros pad the row)
-            for (int l = 0; l <= L; ++l) {
-                const int n = v.n[l], pitch = v.apitch[l];
-                float* dst = v.A + v.aoff[l];
-                for (int e = tid; e < PG * pitch; e += kThreads) {
-                    const int p = e / pitch, i = e - p * pitch;
-                    if (p < np)
-                        dst[(size_t)(p0 + p) * pitch + i] =
-                            (i < n) ? smem[sa[l] + p * n + i] : (i == n ? 1.f : 0.f);
-                }
+            // activation rows, bias column and pads included
+            for (int l = 0; l <= L; ++l)
+                rows_to_global<PG>(v.A + v.aoff[l] + (size_t)p0 * v.apitch[l], smem + q.sa[l],
+                                   v.apitch[l], np);
+            if (Y != nullptr && pr < np) {
+                for (int k = c0; k < nL; k += TP)
+                    Y[(size_t)(p0 + pr) * nL + k] = smem[q.sa[L] + pr * v.apitch[L] + k];
             }
-            if (Y != nullptr) {
-                const int n = v.n[L];
-                for (int e = tid; e < PG * n; e += kThreads) {
-                    const int p = e / n, k = e - p * n;
-                    if (p < np) Y[(size_t)(p0 + p) * n + k] = smem[sa[L] + e];
-                }
-            }
-        } else {
-            for (int l = 1; l <= L; ++l) {
-                const int n = v.n[l], pitch = v.apitch[l];
-                const float* src = v.A + v.aoff[l];
-                for (int e = tid; e < PG * n; e += kThreads) {
-                    const int p = e / n, i = e - p * n;
-                    smem[sa[l] + e] = (p < np) ? __ldcg(src + (size_t)(p0 + p) * pitch + i) : 0.f;
-                }
-            }
-            __syncthreads();
         }
         if (do_bwd) {
             // output delta and error sum (Section 3, fn. 5)
-            for (int e = tid; e < PG * nL; e += kThreads) {
-                const int p = e / nL;
+            const int apL = v.apitch[L], dpL = v.dpitch[L];
+            float* dlt = (L >= 2) ? smem + q.sdt[L] : nullptr;
+            for (int k = c0; k < nL; k += TP) {
                 float d = 0.f;
-                if (p < np) {
-                    const float o = smem[sa[L] + e];
-                    const float err = smem[st + e] - o;
+                if (pr < np) {
+                    const float o = smem[q.sa[L] + pr * apL + k];
+                    const float err = smem[q.st + pr * nL + k] - o;
                     sse = fmaf(err, err, sse);
                     d = err * o * (1.f - o);
                 }
-                smem[sd[L] + e] = d;
+                smem[q.sd[L] + pr * dpL + k] = d;
+                if (dlt != nullptr) dlt[k * PG + pr] = d;
             }
             __syncthreads();
             // hidden deltas, output side first; no delta for the input layer
             for (int l = L - 1; l >= 1; --l) {
-                const int n = v.n[l], nn = v.n[l + 1];
-                const float* Wn = Wb + v.woff[l + 1];
-                for (int i = tid; i < n; i += kThreads) {
-                    float acc[PG];
-#pragma unroll
-                    for (int p = 0; p < PG; ++p) acc[p] = 0.f;
-#pragma unroll 2
-                    for (int j = 0; j < nn; ++j) {
-                        const float w = Wn[(size_t)j * n + i];
-#pragma unroll
-                        for (int p = 0; p < PG; ++p)
-                            acc[p] = fmaf(smem[sd[l + 1] + p * nn + j], w, acc[p]);
-                    }
-#pragma unroll
-                    for (int p = 0; p < PG; ++p) {
-                        const float a = smem[sa[l] + p * n + i];
-                        smem[sd[l] + p * n + i] = acc[p] * a * (1.f - a);
-                    }
-                }
+                hidden_delta<PG>(Wb + v.woff[l + 1], v.kp[l + 1], v.n[l], v.n[l + 1], smem + q.sdt[l + 1],
+                                 smem + q.sa[l], v.apitch[l], smem + q.sd[l], v.dpitch[l],
+                                 l >= 2 ? smem + q.sdt[l] : nullptr, smem + q.red);
                 __syncthreads();
             }
-            for (int l = 1; l <= L; ++l) {
-                const int n = v.n[l], pitch = v.dpitch[l];
-                float* dst = v.D + v.doff[l];
-                for (int e = tid; e < PG * pitch; e += kThreads) {
-                    const int p = e / pitch, i = e - p * pitch;
-                    if (p < np) dst[(size_t)(p0 + p) * pitch + i] = (i < n) ? smem[sd[l] + p * n + i] : 0.f;
-                }
-            }
+            for (int l = 1; l <= L; ++l)
+                rows_to_global<PG>(v.D + v.doff[l] + (size_t)p0 * v.dpitch[l], smem + q.sd[l],
+                                   v.dpitch[l], np);
         }
         __syncthreads();
     }
@@ -491,7 +609,7 @@ __device__ void weight_phase(const F32View& v, int B, bool fused, bool fold_g, f
             for (int s = 0; s < kPS; ++s) g += red[(s * kTU + u) * kTJ + jj];
             const int uu = u0 + u, ii = j0 + jj;
             if (uu < n_out && ii <= n_in) {
-                const long long idx = (ii < n_in) ? v.woff[l] + (long long)uu * n_in + ii : v.boff[l] + uu;
+                const long long idx = v.woff[l] + (long long)uu * v.kp[l] + ii;   // ii == n_in: bias
                 if (!fused) {
                     v.G[idx] += g;
                 } else {
@@ -540,22 +658,22 @@ __device__ void reduce_sse(const F32View& v, int nparts, float* sse_out) {
 // WS: the weights are copied into shared memory (else read from global memory).
 template <int PG, bool WS>
 __global__ void __launch_bounds__(kThreads, 1)
-    k_forward(const __grid_constant__ F32View v, const float* X, int B, float* Y) {
+    k_forward(const __grid_constant__ F32View v, const PatLayout q, const float* X, int B, float* Y) {
     extern __shared__ __align__(128) float smem[];
     __shared__ __align__(8) uint64_t s_bar;
     unsigned phase = 0;
     if (WS) {
         mbar_init1(&s_bar);
         stage_weights(v.theta, v.P, smem, &s_bar, phase, v.flags);
-        pattern_phase<PG>(v, smem, X, nullptr, B, true, false, Y, pattern_base<true>(v, smem));
+        pattern_phase<PG>(v, q, smem, X, nullptr, B, true, false, Y, pattern_base<true>(v, smem));
     } else {
-        pattern_phase<PG>(v, v.theta, X, nullptr, B, true, false, Y, pattern_base<false>(v, smem));
+        pattern_phase<PG>(v, q, v.theta, X, nullptr, B, true, false, Y, pattern_base<false>(v, smem));
     }
 }
 
 template <int PG, bool WS>
 __global__ void __launch_bounds__(kThreads, 1)
-    k_deltas(const __grid_constant__ F32View v, const float* T, int B) {
+    k_deltas(const __grid_constant__ F32View v, const PatLayout q, const float* T, int B) {
     extern __shared__ __align__(128) float smem[];
     __shared__ __align__(8) uint64_t s_bar;
     unsigned phase = 0;
@@ -563,9 +681,9 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (WS) {
         mbar_init1(&s_bar);
         stage_weights(v.theta, v.P, smem, &s_bar, phase, v.flags);
-        e = pattern_phase<PG>(v, smem, nullptr, T, B, false, true, nullptr, pattern_base<true>(v, smem));
+        e = pattern_phase<PG>(v, q, smem, nullptr, T, B, false, true, nullptr, pattern_base<true>(v, smem));
     } else {
-        e = pattern_phase<PG>(v, v.theta, nullptr, T, B, false, true, nullptr, pattern_base<false>(v, smem));
+        e = pattern_phase<PG>(v, q, v.theta, nullptr, T, B, false, true, nullptr, pattern_base<false>(v, smem));
     }
     if (threadIdx.x == 0) v.sse_part[blockIdx.x] = e;
 }
@@ -592,8 +710,8 @@ __global__ void __launch_bounds__(256) k_update(const __grid_constant__ F32View 
 
 template <int PG, bool WS>
 __global__ void __launch_bounds__(kThreads, 1)
-    k_train(const __grid_constant__ F32View v, const float* X, const float* T, int n_patterns,
-            int minibatch, int n_steps, float* sse_out, int fold_g) {
+    k_train(const __grid_constant__ F32View v, const PatLayout q, const float* X, const float* T,
+            int n_patterns, int minibatch, int n_steps, float* sse_out, int fold_g) {
     extern __shared__ __align__(128) float smem[];
     __shared__ __align__(8) uint64_t s_bar;
     __shared__ __align__(8) uint64_t s_cbar[kNBuf];
@@ -617,9 +735,9 @@ __global__ void __launch_bounds__(kThreads, 1)
         float e;
         if (WS) {
             stage_weights(v.theta, v.P, smem, &s_bar, phase, v.flags);
-            e = pattern_phase<PG>(v, smem, Xs, Ts, B, true, true, nullptr, pat);
+            e = pattern_phase<PG>(v, q, smem, Xs, Ts, B, true, true, nullptr, pat);
         } else {
-            e = pattern_phase<PG>(v, v.theta, Xs, Ts, B, true, true, nullptr, pat);
+            e = pattern_phase<PG>(v, q, v.theta, Xs, Ts, B, true, true, nullptr, pat);
         }
         if (threadIdx.x == 0) v.sse_part[blockIdx.x] = e;
         if (!grid_barrier(v.bar, target += gridDim.x, v.flags)) return;
@@ -632,6 +750,35 @@ __global__ void __launch_bounds__(kThreads, 1)
     // every CTA has passed a barrier, so every CTA has read bar[0]: publish the
     // count for the next launch
     if (blockIdx.x == 0 && threadIdx.x == 0) v.bar[0] = target;
+}
+
+// Packed <-> padded parameter layouts, one padded element per thread.
+__device__ __forceinline__ bool padded_source(const F32View& v, long long k, long long& src) {
+    int l = 1;
+    while (l < v.L && k >= v.woff[l + 1]) ++l;
+    const long long r = k - v.woff[l];
+    const int j = (int)(r / v.kp[l]), i = (int)(r - (long long)j * v.kp[l]);
+    const int ni = v.n[l - 1];
+    if (i < ni) src = v.pw[l] + (long long)j * ni + i;
+    else if (i == ni) src = v.pb[l] + j;
+    else return false;
+    return true;
+}
+
+__global__ void __launch_bounds__(256) k_pad(const __grid_constant__ F32View v, const float* packed,
+                                             float* padded) {
+    for (long long k = blockIdx.x * 256LL + threadIdx.x; k < v.P; k += (long long)gridDim.x * 256) {
+        long long src;
+        padded[k] = padded_source(v, k, src) ? packed[src] : 0.f;
+    }
+}
+
+__global__ void __launch_bounds__(256) k_unpad(const __grid_constant__ F32View v, const float* padded,
+                                               float* packed) {
+    for (long long k = blockIdx.x * 256LL + threadIdx.x; k < v.P; k += (long long)gridDim.x * 256) {
+        long long src;
+        if (padded_source(v, k, src)) packed[src] = padded[k];
+    }
 }
 
 template <int PG, bool WS>
@@ -674,11 +821,15 @@ long long f32_layout(F32View& v, const int* n, int L, int cap) {
         v.aoff[l] = a;
         a += (long long)cap * v.apitch[l];
     }
+    long long pp = 0;
     for (int l = 1; l <= L; ++l) {
+        v.kp[l] = v.apitch[l - 1];
         v.woff[l] = pos;
-        pos += (long long)n[l] * n[l - 1];
-        v.boff[l] = pos;
-        pos += n[l];
+        pos += (long long)n[l] * v.kp[l];
+        v.pw[l] = pp;
+        pp += (long long)n[l] * n[l - 1];
+        v.pb[l] = pp;
+        pp += n[l];
         v.dpitch[l] = (n[l] + 3) & ~3;
         v.doff[l] = d;
         d += (long long)cap * v.dpitch[l];
@@ -688,19 +839,52 @@ long long f32_layout(F32View& v, const int* n, int L, int cap) {
         tiles += rows * cols;
         v.tile0[l + 1] = tiles;
     }
-    v.P = pos;
-    v.wsm = (int)((pos + 3) & ~3LL);
+    v.P = pos;   // a multiple of 4: every kp is
+    v.Pp = pp;
+    v.wsm = (int)pos;
     v.a_floats = a;
     v.d_floats = d;
     return a + d;
 }
 
-static size_t pattern_floats(const int* n, int L, int pg) {
-    size_t units = 0;
-    for (int l = 0; l <= L; ++l) units += (size_t)n[l];
-    for (int l = 1; l <= L; ++l) units += (size_t)n[l];
-    units += (size_t)n[L];   // target rows
-    return units * (size_t)pg;
+// Pattern buffers of a CTA for a group size (see PatLayout).
+static PatLayout pat_layout(const int* n, int L, int pg) {
+    PatLayout q{};
+    int off = 0;
+    for (int l = 0; l <= L; ++l) { q.sa[l] = off; off += pg * ((n[l] + 1 + 3) & ~3); }
+    for (int l = 1; l <= L; ++l) { q.sd[l] = off; off += pg * ((n[l] + 3) & ~3); }
+    for (int l = 2; l <= L; ++l) { q.sdt[l] = off; off += (pg * n[l] + 3) & ~3; }
+    q.st = off;
+    off += (pg * n[L] + 3) & ~3;
+    q.red = off;
+    off += kThreads * pg;
+    q.total = off;
+    return q;
+}
+
+static size_t pattern_floats(const int* n, int L, int pg) { return (size_t)pat_layout(n, L, pg).total; }
+
+void f32_pad_host(const F32View& v, const float* packed, float* padded) {
+    for (long long k = 0; k < v.P; ++k) padded[k] = 0.f;
+    for (int l = 1; l <= v.L; ++l) {
+        const int ni = v.n[l - 1];
+        for (int j = 0; j < v.n[l]; ++j) {
+            float* row = padded + v.woff[l] + (long long)j * v.kp[l];
+            for (int i = 0; i < ni; ++i) row[i] = packed[v.pw[l] + (long long)j * ni + i];
+            row[ni] = packed[v.pb[l] + j];
+        }
+    }
+}
+
+void f32_unpad_host(const F32View& v, const float* padded, float* packed) {
+    for (int l = 1; l <= v.L; ++l) {
+        const int ni = v.n[l - 1];
+        for (int j = 0; j < v.n[l]; ++j) {
+            const float* row = padded + v.woff[l] + (long long)j * v.kp[l];
+            for (int i = 0; i < ni; ++i) packed[v.pw[l] + (long long)j * ni + i] = row[i];
+            packed[v.pb[l] + j] = row[ni];
+        }
+    }
 }
 
 // Without the weights in shared memory: the pattern buffers and the
@@ -767,14 +951,15 @@ F32Plan f32_plan(const F32View& v, int batch, int num_sms) {
     size_t need = p.w_in_smem ? (size_t)v.wsm + pat : pat;
     if (need < (size_t)kGradFloats) need = kGradFloats;
     p.smem = need * sizeof(float);
+    p.q = pat_layout(v.n, v.L, pg);
     return p;
 }
 
 cudaError_t f32_forward(const F32View& v, const float* X, int batch, float* Y, const F32Plan& plan,
                         cudaStream_t s) {
 #define BP_FWD(PG)                                                                        \
-    (plan.w_in_smem ? (k_forward<PG, true><<<plan.grid, kThreads, plan.smem, s>>>(v, X, batch, Y)) \
-                    : (k_forward<PG, false><<<plan.grid, kThreads, plan.smem, s>>>(v, X, batch, Y)))
+    (plan.w_in_smem ? (k_forward<PG, true><<<plan.grid, kThreads, plan.smem, s>>>(v, plan.q, X, batch, Y)) \
+                    : (k_forward<PG, false><<<plan.grid, kThreads, plan.smem, s>>>(v, plan.q, X, batch, Y)))
     switch (plan.pg) {
         case 1: BP_FWD(1); break;
         case 2: BP_FWD(2); break;
@@ -788,8 +973,8 @@ cudaError_t f32_forward(const F32View& v, const float* X, int batch, float* Y, c
 cudaError_t f32_backward(const F32View& v, const float* /*X*/, const float* T, int batch,
                          float* sse_out, const F32Plan& plan, cudaStream_t s) {
 #define BP_DEL(PG)                                                                      \
-    (plan.w_in_smem ? (k_deltas<PG, true><<<plan.grid, kThreads, plan.smem, s>>>(v, T, batch)) \
-                    : (k_deltas<PG, false><<<plan.grid, kThreads, plan.smem, s>>>(v, T, batch)))
+    (plan.w_in_smem ? (k_deltas<PG, true><<<plan.grid, kThreads, plan.smem, s>>>(v, plan.q, T, batch)) \
+                    : (k_deltas<PG, false><<<plan.grid, kThreads, plan.smem, s>>>(v, plan.q, T, batch)))
     switch (plan.pg) {
         case 1: BP_DEL(1); break;
         case 2: BP_DEL(2); break;
@@ -802,6 +987,23 @@ cudaError_t f32_backward(const F32View& v, const float* /*X*/, const float* T, i
     const int tiles = v.tile0[v.L + 1];
     const int ggrid = tiles < plan.grid ? tiles : plan.grid;
     k_accumulate<<<ggrid, kThreads, kGradFloats * sizeof(float), s>>>(v, batch, plan.grid, sse_out);
+    return cudaGetLastError();
+}
+
+static int elementwise_blocks(long long n) {
+    long long blocks = (n + 255) / 256;
+    if (blocks > 4096) blocks = 4096;
+    if (blocks < 1) blocks = 1;
+    return (int)blocks;
+}
+
+cudaError_t f32_pad_device(const F32View& v, const float* packed, float* padded, cudaStream_t s) {
+    k_pad<<<elementwise_blocks(v.P), 256, 0, s>>>(v, packed, padded);
+    return cudaGetLastError();
+}
+
+cudaError_t f32_unpad_device(const F32View& v, const float* padded, float* packed, cudaStream_t s) {
+    k_unpad<<<elementwise_blocks(v.P), 256, 0, s>>>(v, padded, packed);
     return cudaGetLastError();
 }
 
@@ -818,7 +1020,8 @@ cudaError_t f32_train(const F32View& v, const float* X, const float* T, int n_pa
                       const F32Plan& plan, cudaStream_t s) {
     int fold = fold_g ? 1 : 0;
     F32View vv = v;
-    void* args[] = {(void*)&vv, (void*)&X, (void*)&T, (void*)&n_patterns, (void*)&minibatch,
+    PatLayout q = plan.q;
+    void* args[] = {(void*)&vv, (void*)&q, (void*)&X, (void*)&T, (void*)&n_patterns, (void*)&minibatch,
                     (void*)&n_steps, (void*)&sse_out, (void*)&fold};
     const void* fn;
     const bool ws = plan.w_in_smem != 0;

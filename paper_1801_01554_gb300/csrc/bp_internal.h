@@ -20,8 +20,13 @@ constexpr int kFlagNonfinite = 2;   // an error sum was NaN/Inf
 constexpr int kBarWords = 4;
 
 // Device view of a float32 net, passed to kernels by value.
-//   theta/V/G: flat parameter vectors (layer order, W_l row-major then b_l),
-//              P values; wsm = P rounded up to 4 (its shared-memory copy).
+//   theta/V/G: flat parameter vectors in the padded device layout: layer by
+//              layer, W_l as [n_l][kp_l] rows with kp_l = apitch_{l-1}, where
+//              column n_{l-1} holds the bias b_l (the true unit's weight) and
+//              the columns after it are zero; P floats in all, a multiple of 4
+//              (also the size of its shared-memory copy, wsm).  The API's
+//              packed layout (W_l row-major, then b_l; Pp floats) is converted
+//              on the way in and out.
 //   A: activation rows of layers 0..L, layer l at aoff[l] with pitch apitch[l]
 //      = n_l + 1 rounded up to 4 (column n_l holds the true unit's 1).
 //   D: delta rows of layers 1..L at doff[l], pitch dpitch[l] = n_l rounded up to 4.
@@ -32,9 +37,12 @@ struct F32View {
     int L;
     int cap;
     int n[BP_MAX_SIZES];
-    long long woff[BP_MAX_SIZES];
-    long long boff[BP_MAX_SIZES];
-    long long P;
+    int kp[BP_MAX_SIZES];          // row pitch of W_l in the padded layout
+    long long woff[BP_MAX_SIZES];  // padded offset of W_l
+    long long pw[BP_MAX_SIZES];    // packed offset of W_l
+    long long pb[BP_MAX_SIZES];    // packed offset of b_l
+    long long P;                   // padded parameter count
+    long long Pp;                  // packed parameter count
     int wsm;
     int apitch[BP_MAX_SIZES];
     int dpitch[BP_MAX_SIZES];
@@ -61,12 +69,28 @@ struct F32View {
     CUtensorMap tm_a[BP_MAX_SIZES];
 };
 
+// Offsets (floats, each a multiple of 4) of a CTA's pattern buffers for PG
+// patterns, computed on the host: activation rows sa[l] ([PG][apitch_l],
+// l = 0..L), delta rows sd[l] ([PG][dpitch_l], l = 1..L), the same deltas
+// pattern-minor sdt[l] ([n_l][PG], l = 2..L, read by the hidden deltas below
+// them), target rows st ([PG][n_L]) and hidden-delta partial sums red
+// (kThreads * PG floats); `total` floats in all.
+struct PatLayout {
+    int sa[BP_MAX_SIZES];
+    int sd[BP_MAX_SIZES];
+    int sdt[BP_MAX_SIZES];
+    int st;
+    int red;
+    int total;
+};
+
 // Launch geometry chosen on the host for a group size.
 struct F32Plan {
     int pg;          // patterns per CTA pass (1, 2, 4 or 8)
     int grid;        // CTAs of the launch
     int w_in_smem;   // the weights are copied into shared memory
     size_t smem;     // dynamic shared memory bytes
+    PatLayout q;     // pattern buffers
 };
 
 // --- float32 path (bp_f32.cu) -------------------------------------------
@@ -86,6 +110,11 @@ cudaError_t f32_forward(const F32View& v, const float* X, int batch, float* Y,
 cudaError_t f32_backward(const F32View& v, const float* X, const float* T, int batch,
                          float* sse_out, const F32Plan& plan, cudaStream_t s);
 cudaError_t f32_update(const F32View& v, long long n_params, cudaStream_t s);
+// Packed <-> padded parameter layouts (see F32View), on the host and on the device.
+void f32_pad_host(const F32View& v, const float* packed, float* padded);
+void f32_unpad_host(const F32View& v, const float* padded, float* packed);
+cudaError_t f32_pad_device(const F32View& v, const float* packed, float* padded, cudaStream_t s);
+cudaError_t f32_unpad_device(const F32View& v, const float* padded, float* packed, cudaStream_t s);
 // Persistent cooperative launch running `n_steps` groups of `minibatch` patterns
 // (the last may be ragged), one update after each.  fold_g: G holds a pending
 // change to add into the first update.

@@ -102,11 +102,12 @@ extern "C" bp_status bp_train_epoch_noalloc(const int* layer_sizes, int n_layers
     if (st != BP_OK) return st;
 
     // scratch layout (floats, each part 16-byte aligned):
-    // [error word, pad][barrier words][per-CTA error sums, padded][activation rows][delta rows]
+    // [error word, pad][barrier words][per-CTA error sums, padded]
+    // [weights, padded layout][weight changes, padded layout][activation rows][delta rows]
     F32View v{};
     const long long soff = f32_layout(v, layer_sizes, L, minibatch);
     const long long bar_words = kBarWords;
-    const long long head = 4 + bar_words + (((long long)sms + 3) & ~3LL);
+    const long long head = 4 + bar_words + (((long long)sms + 3) & ~3LL) + 2 * v.P;
     const long long need = head + soff;
     if (need > (long long)kNoallocScratchFloats) {
         snprintf(msg, sizeof msg,
@@ -119,14 +120,18 @@ extern "C" bp_status bp_train_epoch_noalloc(const int* layer_sizes, int n_layers
     v.flags = reinterpret_cast<int*>(base);
     v.bar = reinterpret_cast<unsigned*>(base + 4);
     v.sse_part = base + 4 + bar_words;
+    float* theta_pad = base + 4 + bar_words + (((long long)sms + 3) & ~3LL);
+    float* V_pad = theta_pad + v.P;
     v.A = base + head;
     v.D = base + head + v.a_floats;
     if (f32_maps(v) != cudaSuccess) {
         set_error_message("bp_train_epoch_noalloc: cuTensorMapEncodeTiled failed for the scratch");
         return BP_ECUDA;
     }
-    v.theta = d_theta;
-    v.V = d_V;
+    // the kernel works on padded copies of the caller's (packed) weights and
+    // weight changes, copied back when it is done
+    v.theta = theta_pad;
+    v.V = V_pad;
     v.G = nullptr;   // nothing pending: the launch never reads G
     v.lr = lr;
     v.momentum = momentum;
@@ -136,11 +141,15 @@ extern "C" bp_status bp_train_epoch_noalloc(const int* layer_sizes, int n_layers
     // the array keeps the last call's contents: the error word and the barrier
     // must start at zero
     cudaError_t e = cudaMemsetAsync(base, 0, (size_t)(4 + bar_words) * sizeof(float), s);
+    if (e == cudaSuccess) e = f32_pad_device(v, d_theta, theta_pad, s);
+    if (e == cudaSuccess) e = f32_pad_device(v, d_V, V_pad, s);
     if (e == cudaSuccess) {
         const F32Plan plan = f32_plan(v, minibatch, sms);
         const int n_steps = (int)(((long long)n_patterns + minibatch - 1) / minibatch);
         e = f32_train(v, d_X, d_T, n_patterns, minibatch, n_steps, d_sse, false, plan, s);
     }
+    if (e == cudaSuccess) e = f32_unpad_device(v, theta_pad, d_theta, s);
+    if (e == cudaSuccess) e = f32_unpad_device(v, V_pad, d_V, s);
     if (e == cudaSuccess && d_status != nullptr)
         e = cudaMemcpyAsync(d_status, base, sizeof(int), cudaMemcpyDeviceToDevice, s);
     if (e != cudaSuccess) {
