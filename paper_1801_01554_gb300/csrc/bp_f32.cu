@@ -145,10 +145,9 @@ __device__ __forceinline__ bool mbar_wait(uint64_t* bar, unsigned parity, int* f
     }
 }
 
-// Copies theta[0, P) into shared memory Ws (one bulk copy for the 16-byte
-// aligned part, plain loads for the tail).  Bounded wait on the mbarrier.
-__device__ void stage_weights(const float* theta, long long P, float* Ws, uint64_t* bar,
-                              unsigned& phase, int* flags) {
+// Starts the copy of theta[0, P) into shared memory Ws: one bulk copy on the
+// mbarrier for the 16-byte aligned part (thread 0), plain loads for the tail.
+__device__ void stage_weights_issue(const float* theta, long long P, float* Ws, uint64_t* bar) {
     const long long P16 = P & ~3LL;
     if (threadIdx.x == 0 && P16 > 0) {
         asm volatile("fence.proxy.async.global;" ::: "memory");
@@ -164,10 +163,26 @@ __device__ void stage_weights(const float* theta, long long P, float* Ws, uint64
             : "memory");
     }
     for (long long k = P16 + threadIdx.x; k < P; k += kThreads) Ws[k] = __ldcg(theta + k);
-    if (P16 > 0) {
-        mbar_wait(bar, phase, flags);
-        phase ^= 1u;
+}
+
+// Bounded wait for a copy started by stage_weights_issue (every thread; the
+// tail written by plain stores needs a CTA barrier after this).
+struct WeightCopy {
+    uint64_t* bar;
+    unsigned* phase;
+    long long P;
+};
+__device__ __forceinline__ void stage_weights_wait(const WeightCopy& w, int* flags) {
+    if ((w.P & ~3LL) > 0) {
+        mbar_wait(w.bar, *w.phase, flags);
+        *w.phase ^= 1u;
     }
+}
+
+__device__ void stage_weights(const float* theta, long long P, float* Ws, uint64_t* bar,
+                              unsigned& phase, int* flags) {
+    stage_weights_issue(theta, P, Ws, bar);
+    stage_weights_wait(WeightCopy{bar, &phase, P}, flags);
     __syncthreads();
 }
 
@@ -253,7 +268,7 @@ __device__ __forceinline__ float4 ld4(const float* p) { return *reinterpret_cast
 // Units per lane group of the forward pass for a group size: every unit's
 // weights are read once per CTA, every activation row once per lane group.
 template <int PG>
-constexpr int fwd_units() { return PG >= 8 ? 4 : 8 / PG; }
+__host__ __device__ constexpr int fwd_units() { return PG >= 8 ? 4 : 8 / PG; }
 
 // Forward through one layer for PG patterns held in shared memory:
 // out[p][j] = sigma(sum_i W[j][i] in[p][i]) over the kp columns of the padded
@@ -426,10 +441,14 @@ __device__ __forceinline__ void rows_to_global(float* dst, const float* src, int
 //   do_bwd: deltas against T, written to scratch
 //   Y: if not null, the outputs are copied there ([B, n_L] packed)
 // Returns this CTA's summed squared error (valid in thread 0).
+//   wc: if not null, a weight copy into shared memory is still in flight; it
+//       is waited for after the first rows have been issued, so that the two
+//       loads overlap
 template <int PG>
 __device__ float pattern_phase(const F32View& v, const PatLayout& q, const float* Wb,
                                const float* __restrict__ X, const float* __restrict__ T, int B,
-                               bool do_fwd, bool do_bwd, float* __restrict__ Y, float* smem) {
+                               bool do_fwd, bool do_bwd, float* __restrict__ Y, float* smem,
+                               const WeightCopy* wc = nullptr) {
     constexpr int TP = kThreads / PG;
     const int L = v.L;
     const int tid = threadIdx.x;
@@ -451,6 +470,10 @@ __device__ float pattern_phase(const F32View& v, const PatLayout& q, const float
                 for (int c = c0; c < q4; c += TP)
                     dst[c] = (pr < np) ? __ldcg(src + c) : make_float4(0.f, 0.f, 0.f, 0.f);
             }
+        }
+        if (wc != nullptr) {
+            stage_weights_wait(*wc, v.flags);
+            wc = nullptr;
         }
         cp_async_wait<0>();
         __syncthreads();
@@ -498,6 +521,7 @@ __device__ float pattern_phase(const F32View& v, const PatLayout& q, const float
         }
         __syncthreads();
     }
+    if (wc != nullptr) stage_weights_wait(*wc, v.flags);   // no patterns here
     // the weight phase reads the activation and delta rows through TMA
     asm volatile("fence.proxy.async.global;" ::: "memory");
     return block_sum(sse);
@@ -734,8 +758,9 @@ __global__ void __launch_bounds__(kThreads, 1)
         const float* Ts = T + p0 * nL;
         float e;
         if (WS) {
-            stage_weights(v.theta, v.P, smem, &s_bar, phase, v.flags);
-            e = pattern_phase<PG>(v, q, smem, Xs, Ts, B, true, true, nullptr, pat);
+            stage_weights_issue(v.theta, v.P, smem, &s_bar);
+            const WeightCopy wc{&s_bar, &phase, v.P};
+            e = pattern_phase<PG>(v, q, smem, Xs, Ts, B, true, true, nullptr, pat, &wc);
         } else {
             e = pattern_phase<PG>(v, q, v.theta, Xs, Ts, B, true, true, nullptr, pat);
         }
