@@ -350,7 +350,12 @@ bp_status bp_update(bp_net* net, void* stream) {
 static bp_status run_epoch(bp_net* net, const void* d_X, const void* d_T, int n_patterns,
                            int minibatch, float* d_sse, cudaStream_t s) {
     const int n_steps = (int)(((long long)n_patterns + minibatch - 1) / minibatch);
-    if (net->dtype == BP_F32) {
+    if (net->dtype == BP_F32 && !net->g_dirty && f32_small_ok(net->view, minibatch)) {
+        // groups of a few patterns: one CTA keeps the weights resident
+        BP_CUDA(f32_train_small(net->view, (const float*)d_X, (const float*)d_T, n_patterns,
+                                minibatch, n_steps, d_sse, s),
+                "training launch");
+    } else if (net->dtype == BP_F32) {
         const F32Plan plan = f32_plan(net->view, minibatch, net->num_sms);
         BP_CUDA(f32_train(net->view, (const float*)d_X, (const float*)d_T, n_patterns, minibatch,
                           n_steps, d_sse, net->g_dirty, plan, s),

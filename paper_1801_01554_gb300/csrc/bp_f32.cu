@@ -444,11 +444,14 @@ __device__ __forceinline__ void rows_to_global(float* dst, const float* src, int
 //   wc: if not null, a weight copy into shared memory is still in flight; it
 //       is waited for after the first rows have been issued, so that the two
 //       loads overlap
+//   to_scratch: write the activation and delta rows to scratch (A, D)
+//   rows_issued: the first pass's rows were already issued (load_rows)
 template <int PG>
 __device__ float pattern_phase(const F32View& v, const PatLayout& q, const float* Wb,
                                const float* __restrict__ X, const float* __restrict__ T, int B,
                                bool do_fwd, bool do_bwd, float* __restrict__ Y, float* smem,
-                               const WeightCopy* wc = nullptr) {
+                               const WeightCopy* wc = nullptr, bool to_scratch = true,
+                               bool rows_issued = false) {
     constexpr int TP = kThreads / PG;
     const int L = v.L;
     const int tid = threadIdx.x;
@@ -459,7 +462,8 @@ __device__ float pattern_phase(const F32View& v, const PatLayout& q, const float
     const int q_hi = (int)((long long)B * (blockIdx.x + 1) / gridDim.x);
     for (int p0 = q_lo; p0 < q_hi; p0 += PG) {
         const int np = min(PG, q_hi - p0);
-        load_rows<PG>(v, q, do_fwd ? X : nullptr, do_bwd ? T : nullptr, p0, np, smem);
+        if (!(rows_issued && p0 == q_lo))
+            load_rows<PG>(v, q, do_fwd ? X : nullptr, do_bwd ? T : nullptr, p0, np, smem);
         if (!do_fwd) {
             // activations of the last forward, reloaded from scratch
             for (int l = 1; l <= L; ++l) {
@@ -484,7 +488,7 @@ __device__ float pattern_phase(const F32View& v, const PatLayout& q, const float
                 __syncthreads();
             }
             // activation rows, bias column and pads included
-            for (int l = 0; l <= L; ++l)
+            for (int l = 0; l <= L && to_scratch; ++l)
                 rows_to_global<PG>(v.A + v.aoff[l] + (size_t)p0 * v.apitch[l], smem + q.sa[l],
                                    v.apitch[l], np);
             if (Y != nullptr && pr < np) {
@@ -515,7 +519,7 @@ __device__ float pattern_phase(const F32View& v, const PatLayout& q, const float
                                  l >= 2 ? smem + q.sdt[l] : nullptr, smem + q.red);
                 __syncthreads();
             }
-            for (int l = 1; l <= L; ++l)
+            for (int l = 1; l <= L && to_scratch; ++l)
                 rows_to_global<PG>(v.D + v.doff[l] + (size_t)p0 * v.dpitch[l], smem + q.sd[l],
                                    v.dpitch[l], np);
         }
@@ -777,6 +781,120 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (blockIdx.x == 0 && threadIdx.x == 0) v.bar[0] = target;
 }
 
+// Online and small-group training on one CTA: Section 3's update after every
+// group of B <= PG patterns (B = 1 is the per-pattern update).  The weights
+// stay in shared memory and the weight changes in registers for the whole
+// launch, so a group costs no grid barrier and no weight copy, and the next
+// group's rows load while this group's update runs (two pattern buffers).
+//
+// Update slots: layer l's padded rows are split into float4 columns c = t % K4
+// (K4 = kp_l / 4) and rows j = t / K4 + R * r (R = kThreads / K4 rows per
+// pass); a thread's slots m in [m0[l], m0[l + 1]) hold the passes r of layer l,
+// so each thread keeps one column of inputs per layer and its changes stay in
+// fixed registers.
+struct SmallPlan {
+    int m0[BP_MAX_SIZES + 1];
+};
+
+template <int PG, int NV4>
+__global__ void __launch_bounds__(kThreads, 1)
+    k_train_small(const __grid_constant__ F32View v, const PatLayout q, const SmallPlan sp,
+                  const float* X, const float* T, int n_patterns, int minibatch, int n_steps,
+                  float* sse_out) {
+    extern __shared__ __align__(128) float smem[];
+    __shared__ __align__(8) uint64_t s_bar;
+    const int tid = threadIdx.x;
+    unsigned phase = 0;
+    mbar_init1(&s_bar);
+    float* pat[2] = {smem + v.wsm, smem + v.wsm + q.total};
+    const int n0 = v.n[0], nL = v.n[v.L];
+    // slot m of this thread: layer lm, row jm (or -1), float4 column cm
+    float4 vel[NV4];
+#pragma unroll
+    for (int m = 0; m < NV4; ++m) {
+        int l = 1;
+        while (l < v.L && m >= sp.m0[l + 1]) ++l;
+        const int K4 = v.kp[l] >> 2, R = kThreads / K4;
+        const int j = tid / K4 + R * (m - sp.m0[l]), c = tid % K4;
+        const bool live = m < sp.m0[v.L + 1] && tid / K4 < R && j < v.n[l];
+        vel[m] = live ? reinterpret_cast<const float4*>(v.V + v.woff[l] + (long long)j * v.kp[l])[c]
+                      : make_float4(0.f, 0.f, 0.f, 0.f);
+    }
+    stage_weights(v.theta, v.P, smem, &s_bar, phase, v.flags);
+    const float a_lr = v.lr * v.grad_scale, mom = v.momentum;
+    if (n_steps > 0)
+        load_rows<PG>(v, q, X, T, 0, (int)min((long long)minibatch, (long long)n_patterns), pat[0]);
+    for (int s = 0; s < n_steps; ++s) {
+        const long long p0 = (long long)s * minibatch;
+        const int B = (int)min((long long)minibatch, (long long)n_patterns - p0);
+        float* ps = pat[s & 1];
+        const float e = pattern_phase<PG>(v, q, smem, X + p0 * n0, T + p0 * nL, B, true, true, nullptr,
+                                          ps, nullptr, false, true);
+        if (tid == 0) {
+            if (sse_out != nullptr) sse_out[s] = e;
+            if (!isfinite(e)) atomicOr(v.flags, kFlagNonfinite);
+        }
+        if (s + 1 < n_steps) {
+            const long long pn = p0 + minibatch;
+            load_rows<PG>(v, q, X + pn * n0, T + pn * nL, 0,
+                          (int)min((long long)minibatch, (long long)n_patterns - pn), pat[(s + 1) & 1]);
+        }
+        // momentum update of every weight from this group's deltas and inputs
+        int l = 0, K4 = 1, c = 0, j0 = 0, R = 1;
+        float4 a[PG];
+#pragma unroll
+        for (int m = 0; m < NV4; ++m) {
+            if (m >= sp.m0[v.L + 1]) break;
+            if (l < v.L && m == sp.m0[l + 1]) {   // next layer: its input column
+                ++l;
+                K4 = v.kp[l] >> 2;
+                R = kThreads / K4;
+                c = tid % K4;
+                j0 = tid / K4;
+#pragma unroll
+                for (int p = 0; p < PG; ++p) a[p] = ld4(ps + q.sa[l - 1] + p * v.apitch[l - 1] + 4 * c);
+            }
+            const int j = j0 + R * (m - sp.m0[l]);
+            if (j0 < R && j < v.n[l]) {
+                float4 g = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+                for (int p = 0; p < PG; ++p) {
+                    const float d = ps[q.sd[l] + p * v.dpitch[l] + j];
+                    g.x = fmaf(d, a[p].x, g.x);
+                    g.y = fmaf(d, a[p].y, g.y);
+                    g.z = fmaf(d, a[p].z, g.z);
+                    g.w = fmaf(d, a[p].w, g.w);
+                }
+                float4* wp = reinterpret_cast<float4*>(smem + v.woff[l] + (long long)j * v.kp[l]) + c;
+                float4 w = *wp;
+                float4& u = vel[m];
+                u.x = a_lr * g.x + mom * u.x;
+                u.y = a_lr * g.y + mom * u.y;
+                u.z = a_lr * g.z + mom * u.z;
+                u.w = a_lr * g.w + mom * u.w;
+                w.x += u.x;
+                w.y += u.y;
+                w.z += u.z;
+                w.w += u.w;
+                *wp = w;
+            }
+        }
+        __syncthreads();
+    }
+    // weights and weight changes back to global memory
+    for (long long k = tid; k < (v.P >> 2); k += kThreads)
+        reinterpret_cast<float4*>(v.theta)[k] = reinterpret_cast<const float4*>(smem)[k];
+#pragma unroll
+    for (int m = 0; m < NV4; ++m) {
+        int l = 1;
+        while (l < v.L && m >= sp.m0[l + 1]) ++l;
+        const int K4 = v.kp[l] >> 2, R = kThreads / K4;
+        const int j = tid / K4 + R * (m - sp.m0[l]), c = tid % K4;
+        if (m < sp.m0[v.L + 1] && tid / K4 < R && j < v.n[l])
+            reinterpret_cast<float4*>(v.V + v.woff[l] + (long long)j * v.kp[l])[c] = vel[m];
+    }
+}
+
 // Packed <-> padded parameter layouts, one padded element per thread.
 __device__ __forceinline__ bool padded_source(const F32View& v, long long k, long long& src) {
     int l = 1;
@@ -949,6 +1067,15 @@ cudaError_t f32_maps(F32View& v) {
     return cudaSuccess;
 }
 
+template <int PG>
+cudaError_t set_small_attr(size_t bytes) {
+    cudaError_t e = cudaFuncSetAttribute(k_train_small<PG, 4>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         (int)bytes);
+    if (e != cudaSuccess) return e;
+    return cudaFuncSetAttribute(k_train_small<PG, 16>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                (int)bytes);
+}
+
 cudaError_t f32_setup(int device) {
     int optin = 0;
     cudaError_t e = cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, device);
@@ -958,6 +1085,9 @@ cudaError_t f32_setup(int device) {
     if ((e = set_smem_attr<2>(kSmemLimit)) != cudaSuccess) return e;
     if ((e = set_smem_attr<4>(kSmemLimit)) != cudaSuccess) return e;
     if ((e = set_smem_attr<8>(kSmemLimit)) != cudaSuccess) return e;
+    if ((e = set_small_attr<1>(kSmemLimit)) != cudaSuccess) return e;
+    if ((e = set_small_attr<2>(kSmemLimit)) != cudaSuccess) return e;
+    if ((e = set_small_attr<4>(kSmemLimit)) != cudaSuccess) return e;
     return cudaFuncSetAttribute(k_accumulate, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                 (int)(kGradFloats * sizeof(float)));
 }
@@ -1057,6 +1187,54 @@ cudaError_t f32_train(const F32View& v, const float* X, const float* T, int n_pa
         default: fn = ws ? (const void*)k_train<8, true> : (const void*)k_train<8, false>; break;
     }
     return cudaLaunchCooperativeKernel(fn, dim3(plan.grid), dim3(kThreads), args, plan.smem, s);
+}
+
+// ------------------------------------------------------------ one-CTA groups
+// Groups of at most kSmallMaxB patterns run on one CTA when the padded weights
+// and the pattern buffers fit in its shared memory and the weight changes fit
+// in its registers (16 float4 per thread).
+constexpr int kSmallMaxB = 4;
+
+// Update slots per thread: layer l takes ceil(n_l / (kThreads / (kp_l / 4))) passes.
+static SmallPlan small_plan(const F32View& v) {
+    SmallPlan sp{};
+    int m = 0;
+    for (int l = 1; l <= v.L; ++l) {
+        sp.m0[l] = m;
+        const int K4 = v.kp[l] / 4;
+        const int R = K4 <= kThreads ? kThreads / K4 : 0;
+        m += R > 0 ? (v.n[l] + R - 1) / R : 1 << 20;
+    }
+    sp.m0[v.L + 1] = m;
+    return sp;
+}
+
+bool f32_small_ok(const F32View& v, int minibatch) {
+    if (minibatch > kSmallMaxB) return false;
+    const int pg = minibatch <= 1 ? 1 : minibatch <= 2 ? 2 : 4;
+    if (small_plan(v).m0[v.L + 1] > 16) return false;
+    const size_t bytes = ((size_t)v.wsm + 2 * (size_t)pat_layout(v.n, v.L, pg).total) * sizeof(float);
+    return bytes <= kSmemLimit;
+}
+
+cudaError_t f32_train_small(const F32View& v, const float* X, const float* T, int n_patterns,
+                            int minibatch, int n_steps, float* sse_out, cudaStream_t s) {
+    if (!f32_small_ok(v, minibatch)) return cudaErrorInvalidValue;
+    const int pg = minibatch <= 1 ? 1 : minibatch <= 2 ? 2 : 4;
+    const PatLayout q = pat_layout(v.n, v.L, pg);
+    const SmallPlan sp = small_plan(v);
+    const size_t bytes = ((size_t)v.wsm + 2 * (size_t)q.total) * sizeof(float);
+    const bool big = sp.m0[v.L + 1] > 4;
+#define BP_SMALL(PG, NV)                                                                        \
+    k_train_small<PG, NV><<<1, kThreads, bytes, s>>>(v, q, sp, X, T, n_patterns, minibatch, n_steps, \
+                                                     sse_out)
+    switch (pg) {
+        case 1: if (big) BP_SMALL(1, 16); else BP_SMALL(1, 4); break;
+        case 2: if (big) BP_SMALL(2, 16); else BP_SMALL(2, 4); break;
+        default: if (big) BP_SMALL(4, 16); else BP_SMALL(4, 4); break;
+    }
+#undef BP_SMALL
+    return cudaGetLastError();
 }
 
 }  // namespace bp

@@ -122,6 +122,13 @@ cudaError_t f32_train(const F32View& v, const float* X, const float* T, int n_pa
                       int minibatch, int n_steps, float* sse_out, bool fold_g,
                       const F32Plan& plan, cudaStream_t s);
 
+// Groups of at most 4 patterns on one CTA, with the weights resident in its
+// shared memory for the whole launch (f32_small_ok says whether the net fits;
+// no pending change G is folded in).
+bool f32_small_ok(const F32View& v, int minibatch);
+cudaError_t f32_train_small(const F32View& v, const float* X, const float* T, int n_patterns,
+                            int minibatch, int n_steps, float* sse_out, cudaStream_t s);
+
 // Message returned by bp_last_error() on the calling thread (bp_api.cu).
 void set_error_message(const char* msg);
 

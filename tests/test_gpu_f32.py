@@ -135,6 +135,34 @@ def test_train_epoch_matches_oracle(n, mb):
         assert normwise(net.get_weights() - theta, st.theta - theta) <= 1e-4
 
 
+@pytest.mark.parametrize("sizes,n,mb", [((203, 120, 26), 300, 1), ((203, 120, 26), 301, 2),
+                                         ((203, 60, 26), 259, 3), ((203, 60, 26), 256, 4),
+                                         ((5, 3, 2), 50, 1), ((64, 33, 17, 9), 130, 4),
+                                         ((40, 300, 200, 1), 64, 2)])
+def test_small_group_epoch_matches_oracle(sizes, n, mb):
+    """Groups of 1-4 patterns (the per-pattern update of Section 3 at mb = 1),
+    ragged last groups, a deep net, and a net too large for one CTA."""
+    X, T, theta = problem(sizes, n, seed=21)
+    V0 = synth.round_to(np.random.default_rng(3).uniform(-1e-3, 1e-3, theta.size), "f32")
+    st = O.State(sizes, theta, lr=0.05, momentum=0.9, V=V0.copy())
+    e_ref = O.train_epoch(st, X, T, mb)
+    runs = []
+    for _ in range(2):
+        with bp.Net(sizes, 0.05, 0.9, bp.BP_F32, max_batch=mb) as net:
+            net.set_weights(theta)
+            net.set_velocity(V0)
+            sse = torch.zeros(len(e_ref), device="cuda")
+            net.train_epoch(dev(X), dev(T), n, mb, sse)
+            net.check()
+            runs.append((net.get_weights(), net.get_velocity(), sse.cpu().numpy()))
+    W1, V1, e1 = runs[0]
+    np.testing.assert_allclose(e1, e_ref, rtol=1e-4, atol=1e-6)
+    assert normwise(W1 - theta, st.theta - theta) <= 1e-4
+    assert normwise(V1, st.V) <= 1e-4
+    # the same launch twice gives the same bits
+    assert np.array_equal(W1, runs[1][0]) and np.array_equal(e1, runs[1][2])
+
+
 @pytest.mark.parametrize("B", synth.SWEEP_BATCHES)
 def test_batch_sweep_step_matches_oracle(B):
     sizes = (203, 120, 26)
