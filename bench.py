@@ -424,6 +424,52 @@ def run_wide(args, world, rank, local):
     return 0
 
 
+# ------------------------------------------------------------------ group-size sweep
+def run_sweep(args, world, rank, local):
+    """CPS against the group size B on the 203-120-26 net (the paper's group-size
+    question, Section 5): one JSON line per B, from CUDA events around whole
+    epochs with the L2 flushed before each.  B <= 4 runs on the one-CTA kernel,
+    larger groups on the persistent kernel."""
+    import torch
+    from paper_1801_01554_gb300 import bp, synth
+
+    if rank != 0:
+        return 0
+    torch.cuda.set_device(local)
+    device = torch.device("cuda", local)
+    sizes = synth.WORKLOADS[WORKLOAD]["sizes"]
+    X, T = synth.nettalk_patterns(65536, seed=0)
+    theta = synth.round_to(synth.init_uniform(sizes, -0.3, 0.3, 0), "f32")
+    Xd = torch.tensor(X, dtype=torch.float32, device=device)
+    Td = torch.tensor(T, dtype=torch.float32, device=device)
+    flush = torch.empty(L2_FLUSH_BYTES // 4, dtype=torch.float32, device=device)
+    W = connections(sizes)
+    for B in (1, 2, 4) + tuple(synth.SWEEP_BATCHES[1:]):
+        n = 65536 if B >= 512 else B * 512          # at least 128 updates per epoch
+        updates = (n + B - 1) // B
+        net = bp.Net(sizes, 0.05, 0.9, bp.BP_F32, max_batch=B)
+        net.set_weights(theta)
+        for _ in range(3):
+            net.train_epoch(Xd, Td, n, B)
+        ms = []
+        for k in range(5):
+            flush.fill_(float(k))
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record()
+            net.train_epoch(Xd, Td, n, B)
+            e1.record()
+            torch.cuda.synchronize(device)
+            ms.append(e0.elapsed_time(e1))
+        net.check()
+        net.close()
+        t = sorted(ms)[len(ms) // 2] / 1e3
+        print(json.dumps({"sweep": "group size", "B": B, "patterns": n, "updates": updates,
+                          "us_per_update": 1e6 * t / updates, "value": W * n / t, "unit": UNIT,
+                          "kernel": "one-CTA" if B <= 4 else "persistent cooperative",
+                          "dtype": "f32", "data": "synthetic"}), flush=True)
+    return 0
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -435,12 +481,16 @@ def main():
     ap.add_argument("--workload", default=WORKLOAD,
                     choices=("nettalk60", "nettalk120", "wide3", "wide4096"),
                     help="workload to time (default: the 203-120-26 NETtalk-shaped net)")
+    ap.add_argument("--sweep", action="store_true",
+                    help="instead of the bench line: CPS against the group size (203-120-26)")
     args = ap.parse_args()
     if args.warmup < 3 and args.impl == "ours":
         args.warmup = 3
     world, rank, local = dist_setup()
     if args.impl == "reference":
         rc = run_reference(args, world, rank)
+    elif args.sweep:
+        rc = run_sweep(args, world, rank, local)
     elif args.workload in ("wide3", "wide4096"):
         rc = run_wide(args, world, rank, local)
     else:
