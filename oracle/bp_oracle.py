@@ -22,7 +22,9 @@ CMU-CS-89-208):
 * pooled update: weight changes are summed over all patterns of a group and
   applied once (Sections 3 and 4.1);
 * the update routine applies the learning rate and momentum to the summed
-  change and zeroes the accumulator (Section 6.2.1).
+  change and zeroes the accumulator (Section 6.2.1);
+* optionally, the table-lookup logistic of Section 4.3 (256 points over
+  [-15, 15], linear interpolation, clamped outside) in place of 1/(1+e^-x).
 
 Readings taken where the paper is silent (each is listed in the design doc):
 
@@ -104,16 +106,51 @@ def sigmoid(x):
     return 1.0 / (1.0 + np.exp(-x))
 
 
-def forward(Ws, bs, X):
+# Table-lookup logistic (Section 4.3, Figure 3): 256 precomputed values of the
+# logistic at equally spaced points over [-15, 15].
+SIGMOID_TABLE_LO = -15.0
+SIGMOID_TABLE_HI = 15.0
+SIGMOID_TABLE_POINTS = 256
+
+
+def sigmoid_table(x):
+    """The second GF11 method of Section 4.3, step by step:
+
+    1. net inputs outside [-15, 15] are mapped to the extreme values of the
+       table (the logistic at -15 and at 15);
+    2. inputs inside are remapped by an addition and a multiplication to x1 in
+       [0, 255];
+    3. the integer part of x1 indexes a table of 1/(1+e^-x) at 256 equally
+       spaced points, and the fractional part interpolates linearly between
+       that entry and the next (at x1 = 255 the last entry is returned).
+    """
+    x = np.asarray(x, dtype=np.float64)
+    n = SIGMOID_TABLE_POINTS
+    nodes = SIGMOID_TABLE_LO + (SIGMOID_TABLE_HI - SIGMOID_TABLE_LO) * np.arange(n) / (n - 1)
+    table = sigmoid(nodes)
+    xc = np.clip(x, SIGMOID_TABLE_LO, SIGMOID_TABLE_HI)
+    x1 = (xc - SIGMOID_TABLE_LO) * ((n - 1) / (SIGMOID_TABLE_HI - SIGMOID_TABLE_LO))
+    i = np.minimum(np.floor(x1), n - 2).astype(np.int64)
+    f = x1 - i
+    return table[i] + f * (table[i + 1] - table[i])
+
+
+SQUASH = {"logistic": sigmoid, "table": sigmoid_table}
+
+
+def forward(Ws, bs, X, squash="logistic"):
     """Activations [A_0 = X, A_1, ..., A_L]; A_l = sigma(A_{l-1} W_l^T + b_l).
 
     Section 3: a unit's activation is the logistic of the weighted sum of the
-    activations connected to it; the bias is the true unit's weight.
+    activations connected to it; the bias is the true unit's weight.  With
+    squash="table" sigma is the table-lookup logistic of Section 4.3; the
+    deltas still use a (1 - a) of the activations it produced.
     """
+    fn = SQUASH[squash]
     As = [np.asarray(X, dtype=np.float64)]
     for W, b in zip(Ws, bs):
         net = As[-1] @ W.T + b[None, :]
-        As.append(sigmoid(net))
+        As.append(fn(net))
     return As
 
 
@@ -172,6 +209,7 @@ class State:
     grad_scale: float = 1.0
     V: np.ndarray = field(default=None)   # previous weight change
     G: np.ndarray = field(default=None)   # pooled change not yet applied
+    squash: str = "logistic"              # or "table" (Section 4.3)
 
     def __post_init__(self):
         self.sizes = tuple(int(s) for s in self.sizes)
@@ -186,7 +224,7 @@ def step_quantities(state: State, X, T):
     """Everything one group of patterns yields: activations, deltas, the pooled
     change (flat, same layout as theta) and the SSE.  Does not modify state."""
     Ws, bs = unpack(state.sizes, state.theta)
-    As = forward(Ws, bs, X)
+    As = forward(Ws, bs, X, state.squash)
     Ds = deltas(Ws, As, T)
     Gs, gs = gradients(As, Ds)
     return As, Ds, pack(Gs, gs), sse(As[-1], T)
@@ -225,4 +263,4 @@ def train_epoch(state: State, X, T, minibatch: int):
 
 def predict(state: State, X):
     Ws, bs = unpack(state.sizes, state.theta)
-    return forward(Ws, bs, X)[-1]
+    return forward(Ws, bs, X, state.squash)[-1]

@@ -242,3 +242,65 @@ def test_bf16_rounding_matches_torch():
     x = np.random.default_rng(0).standard_normal(10000) * 10
     ref = torch.tensor(x, dtype=torch.float32).to(torch.bfloat16).to(torch.float64).numpy()
     np.testing.assert_array_equal(synth.bf16_round(x), ref)
+
+
+# ---------------------------------------------------------------- table sigmoid (Section 4.3)
+def _table_nodes():
+    # 256 points spread evenly over [-15, 15] (Section 4.3, Figure 3)
+    return np.linspace(-15.0, 15.0, 256)
+
+
+def test_sigmoid_table_is_exact_at_its_points():
+    x = _table_nodes()
+    np.testing.assert_allclose(O.sigmoid_table(x), expit(x), rtol=0, atol=1e-15)
+
+
+def test_sigmoid_table_interpolates_linearly_between_points():
+    x = _table_nodes()
+    for k in (0, 17, 127, 128, 200, 254):
+        for t in (0.25, 0.5, 0.9):
+            xm = x[k] + t * (x[k + 1] - x[k])
+            want = expit(x[k]) + t * (expit(x[k + 1]) - expit(x[k]))
+            assert abs(O.sigmoid_table(xm) - want) <= 1e-13
+
+
+def test_sigmoid_table_error_bound():
+    # linear interpolation error <= h^2/8 max|s''| with h = 30/255 and
+    # max|s''| = 1/(6 sqrt 3) (at s = 1/2 -/+ 1/(2 sqrt 3)); outside [-15, 15]
+    # the error is at most s(-15).  The bound is nearly reached near the
+    # inflections of s', so the grid's worst case sits just below it.
+    h = 30.0 / 255.0
+    bound = h * h / 8.0 / (6.0 * math.sqrt(3.0))
+    x = np.linspace(-25.0, 25.0, 2_000_001)
+    err = np.abs(O.sigmoid_table(x) - expit(x))
+    assert err.max() <= bound
+    assert err.max() >= 0.97 * bound
+    assert 1.6e-4 < bound < 1.7e-4
+
+
+def test_sigmoid_table_clamps_to_its_end_values():
+    for x, end in ((40.0, 15.0), (-40.0, -15.0), (15.0, 15.0), (-15.0, -15.0)):
+        assert O.sigmoid_table(x) == pytest.approx(expit(end), abs=1e-16)
+
+
+def test_sigmoid_table_is_odd_about_one_half_and_monotone():
+    x = np.random.default_rng(5).uniform(-20, 20, 10_000)
+    np.testing.assert_allclose(O.sigmoid_table(-x) + O.sigmoid_table(x), 1.0, rtol=0, atol=1e-15)
+    g = np.linspace(-16, 16, 100_001)
+    assert np.all(np.diff(O.sigmoid_table(g)) >= 0)
+
+
+def test_table_squash_changes_a_step_by_at_most_its_error():
+    # one training step with the table logistic against the exact one: the
+    # outputs differ by no more than the table's error bound propagated through
+    # a 2-layer net of small weights (a loose, order-of-magnitude pin)
+    sizes = (203, 60, 26)
+    X, T = synth.nettalk_patterns(64, seed=3)
+    theta = synth.init_uniform(sizes, -0.3, 0.3, 3)
+    a = O.State(sizes, theta, lr=0.05, momentum=0.9)
+    b = O.State(sizes, theta, lr=0.05, momentum=0.9, squash="table")
+    ya, yb = O.predict(a, X), O.predict(b, X)
+    assert 0 < np.abs(ya - yb).max() < 1e-3
+    O.train_batch(a, X, T)
+    O.train_batch(b, X, T)
+    assert np.abs(a.theta - b.theta).max() < 1e-3
