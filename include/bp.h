@@ -87,6 +87,20 @@ void bp_destroy(bp_net* net);
  * after the call.  Errors: BP_EINVAL if a value is not finite. */
 bp_status bp_set_hparams(bp_net* net, float lr, float momentum, float grad_scale);
 
+/* Squashing function of the forward pass (Section 4.3, Figure 3).
+ *   BP_SIGMOID_LOGISTIC (default): 1 / (1 + e^-x), with CUDA's expf.
+ *   BP_SIGMOID_TABLE: the GF11's table-lookup logistic: net inputs outside
+ *     [-15, 15] take the logistic at -15 or 15; inside, the input is remapped
+ *     to [0, 255], its integer part picks one of 256 precomputed values of the
+ *     logistic at equally spaced points and its fractional part interpolates
+ *     linearly to the next one.  Its error against the logistic is at most
+ *     h^2/8 * max|s''| = 1.66e-4 (h = 30/255).  The deltas use a (1 - a) of the
+ *     activations it produces.
+ * Takes effect for work queued after the call.  Errors: BP_EINVAL for an
+ * unknown mode, or BP_SIGMOID_TABLE on a BP_BF16 net (float32 nets only). */
+enum { BP_SIGMOID_LOGISTIC = 0, BP_SIGMOID_TABLE = 1 };
+bp_status bp_set_sigmoid(bp_net* net, int mode);
+
 /* Number of float32 values in a parameter vector (W and b of every layer). */
 int64_t bp_num_params(const bp_net* net);
 

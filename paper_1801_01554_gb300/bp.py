@@ -19,6 +19,7 @@ BP_OK, BP_EINVAL, BP_ENOMEM, BP_ECUDA, BP_ESHAPE, BP_ETIMEOUT, BP_ENONFINITE, BP
 STATUS_NAMES = ["BP_OK", "BP_EINVAL", "BP_ENOMEM", "BP_ECUDA", "BP_ESHAPE", "BP_ETIMEOUT",
                 "BP_ENONFINITE", "BP_ESTATE"]
 BP_F32, BP_BF16 = 0, 1
+BP_SIGMOID_LOGISTIC, BP_SIGMOID_TABLE = 0, 1
 BP_MAX_SIZES = 9
 
 # name -> (restype, argtypes); every symbol declared in include/bp.h
@@ -30,6 +31,7 @@ SIGNATURES = {
     "bp_create": (_I, [ctypes.POINTER(_I), _I, _F, _F, _I, _I, ctypes.POINTER(_VP)]),
     "bp_destroy": (None, [_VP]),
     "bp_set_hparams": (_I, [_VP, _F, _F, _F]),
+    "bp_set_sigmoid": (_I, [_VP, _I]),
     "bp_num_params": (ctypes.c_int64, [_VP]),
     "bp_set_weights": (_I, [_VP, _FP]),
     "bp_get_weights": (_I, [_VP, _FP]),
@@ -141,6 +143,10 @@ def bp_destroy(h):
 
 def bp_set_hparams(h, lr, momentum, grad_scale=1.0):
     _check(load().bp_set_hparams(h, float(lr), float(momentum), float(grad_scale)))
+
+
+def bp_set_sigmoid(h, mode):
+    _check(load().bp_set_sigmoid(h, int(mode)))
 
 
 def bp_num_params(h) -> int:
@@ -263,6 +269,9 @@ class Net:
 
     def set_hparams(self, lr, momentum, grad_scale=1.0):
         bp_set_hparams(self.h, lr, momentum, grad_scale)
+
+    def set_sigmoid(self, mode):
+        bp_set_sigmoid(self.h, mode)
 
     def set_weights(self, theta):
         bp_set_weights(self.h, theta)

@@ -244,6 +244,16 @@ bp_status bp_set_hparams(bp_net* net, float lr, float momentum, float grad_scale
     return BP_OK;
 }
 
+bp_status bp_set_sigmoid(bp_net* net, int mode) {
+    if (net == nullptr) return fail(BP_EINVAL, "NULL net");
+    if (mode != BP_SIGMOID_LOGISTIC && mode != BP_SIGMOID_TABLE)
+        return fail(BP_EINVAL, "unknown sigmoid mode %d", mode);
+    if (mode == BP_SIGMOID_TABLE && net->dtype != BP_F32)
+        return fail(BP_EINVAL, "the table-lookup sigmoid is implemented for float32 nets only");
+    net->view.sig_table = mode == BP_SIGMOID_TABLE ? 1 : 0;
+    return BP_OK;
+}
+
 int64_t bp_num_params(const bp_net* net) { return net ? (int64_t)net->P : 0; }
 
 // Copies a parameter vector between the caller's packed layout (host) and the

@@ -49,6 +49,30 @@ constexpr unsigned kWaitIters = 1u << 26;
 // ------------------------------------------------------------ small helpers
 __device__ __forceinline__ float sigmoid_f(float x) { return 1.0f / (1.0f + expf(-x)); }
 
+// Table-lookup logistic (Section 4.3, Figure 3): the logistic at 256 equally
+// spaced points over [-15, 15], built in shared memory by each CTA that runs a
+// forward pass with the table mode on.  Inputs outside the range take the end
+// values; inside, x is remapped to [0, 255], the integer part picks the entry
+// and the fractional part interpolates linearly to the next one.  NaN stays NaN.
+constexpr int kSigPoints = 256;
+__shared__ float s_sigtab[kSigPoints];
+
+__device__ void sigmoid_table_init(const F32View& v) {
+    if (v.sig_table)
+        for (int k = threadIdx.x; k < kSigPoints; k += blockDim.x)
+            s_sigtab[k] = sigmoid_f(-15.f + (30.f * (float)k) / (float)(kSigPoints - 1));
+}
+
+__device__ __forceinline__ float sigmoid_tab(float x) {
+    if (x != x) return x;
+    const float xc = fminf(fmaxf(x, -15.f), 15.f);
+    const float x1 = (xc + 15.f) * ((float)(kSigPoints - 1) / 30.f);
+    const int i = min((int)x1, kSigPoints - 2);   // x1 >= 0: truncation is the floor
+    const float f = x1 - (float)i;
+    const float t0 = s_sigtab[i];
+    return fmaf(f, s_sigtab[i + 1] - t0, t0);
+}
+
 __device__ __forceinline__ unsigned ld_acquire(const unsigned* p) {
     unsigned v;
     asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
@@ -279,7 +303,7 @@ __host__ __device__ constexpr int fwd_units() { return PG >= 8 ? 4 : 8 / PG; }
 // blocks.
 template <int PG>
 __device__ void forward_layer(const float* W, int kp, int n_out, const float* s_in, float* s_out,
-                              int kp_out) {
+                              int kp_out, bool table) {
     constexpr int U = fwd_units<PG>();
     constexpr int V = U * PG;
     static_assert(V <= 32, "a lane group holds at most 32 sums");
@@ -325,7 +349,7 @@ __device__ void forward_layer(const float* W, int kp, int n_out, const float* s_
         if (s < V && g < G) {
             const int u = s / PG, p = s % PG;
             const int j = j0 + u;
-            if (j < n_out) s_out[p * kp_out + j] = sigmoid_f(r);
+            if (j < n_out) s_out[p * kp_out + j] = table ? sigmoid_tab(r) : sigmoid_f(r);
         }
     }
 }
@@ -484,7 +508,7 @@ __device__ float pattern_phase(const F32View& v, const PatLayout& q, const float
         if (do_fwd) {
             for (int l = 1; l <= L; ++l) {
                 forward_layer<PG>(Wb + v.woff[l], v.kp[l], v.n[l], smem + q.sa[l - 1], smem + q.sa[l],
-                                  v.apitch[l]);
+                                  v.apitch[l], v.sig_table != 0);
                 __syncthreads();
             }
             // activation rows, bias column and pads included
@@ -690,6 +714,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     extern __shared__ __align__(128) float smem[];
     __shared__ __align__(8) uint64_t s_bar;
     unsigned phase = 0;
+    sigmoid_table_init(v);
+    __syncthreads();
     if (WS) {
         mbar_init1(&s_bar);
         stage_weights(v.theta, v.P, smem, &s_bar, phase, v.flags);
@@ -747,6 +773,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     // nothing until bp_check() has cleared the latch and reset the barrier.
     if (__ldcg(v.flags) & kFlagTimeout) return;
     unsigned phase = 0;
+    sigmoid_table_init(v);
     mbar_init1(&s_bar);
     ChunkPipe pipe;
     pipe_init(pipe, s_cbar);
@@ -805,6 +832,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     __shared__ __align__(8) uint64_t s_bar;
     const int tid = threadIdx.x;
     unsigned phase = 0;
+    sigmoid_table_init(v);
     mbar_init1(&s_bar);
     float* pat[2] = {smem + v.wsm, smem + v.wsm + q.total};
     const int n0 = v.n[0], nL = v.n[v.L];
@@ -949,7 +977,7 @@ cudaError_t set_smem_attr(size_t bytes) {
 // ------------------------------------------------------------ host side
 // Dynamic shared memory a CTA may use: the opt-in limit (227 KB on sm_103a)
 // minus room for the kernels' static shared arrays.
-constexpr size_t kStaticSmemReserve = 1024;
+constexpr size_t kStaticSmemReserve = 2048;
 constexpr size_t kSmemLimit = 227 * 1024 - kStaticSmemReserve;
 
 long long f32_layout(F32View& v, const int* n, int L, int cap) {

@@ -60,6 +60,7 @@ struct F32View {
     unsigned* bar;        // grid barrier: [0] count at the end of the last launch, [1] arrival count
     int* flags;           // latched error bits
     float lr, momentum, grad_scale;
+    int sig_table;        // 1: table-lookup logistic (Section 4.3) in the forward pass
     // TMA maps of the weight phase (f32_maps): tm_d[l] over the delta rows of
     // layer l (boxes of 8 columns x 256 patterns), tm_a[l] over the activation
     // rows of layer l (boxes of 32 columns x 256 patterns); zero fill past the

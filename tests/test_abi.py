@@ -70,4 +70,5 @@ def test_null_handles_are_rejected(lib):
     assert lib.bp_forward(None, None, 1, None, None) == bp.BP_EINVAL
     assert lib.bp_check(None, None) == bp.BP_EINVAL
     assert lib.bp_num_params(None) == 0
+    assert lib.bp_set_sigmoid(None, bp.BP_SIGMOID_TABLE) == bp.BP_EINVAL
     lib.bp_destroy(None)   # NULL-safe

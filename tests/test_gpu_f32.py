@@ -163,6 +163,48 @@ def test_small_group_epoch_matches_oracle(sizes, n, mb):
     assert np.array_equal(W1, runs[1][0]) and np.array_equal(e1, runs[1][2])
 
 
+@pytest.mark.parametrize("sizes,n,mb", [((203, 120, 26), 1024, 512), ((203, 60, 26), 300, 1),
+                                         ((203, 60, 26), 301, 4), ((64, 33, 17, 9), 257, 256)])
+def test_table_sigmoid_matches_oracle(sizes, n, mb):
+    """The table-lookup logistic of Section 4.3 on both float32 kernels: the
+    outputs of a forward pass and an epoch of updates against the oracle's
+    table mode; the mode is per net and switches back to the logistic."""
+    X, T, theta = problem(sizes, n, seed=31, lo=-1.0, hi=1.0)
+    st = O.State(sizes, theta, lr=0.05, momentum=0.9, squash="table")
+    Y_ref = O.predict(st, X)
+    e_ref = O.train_epoch(st, X, T, mb)
+    with bp.Net(sizes, 0.05, 0.9, bp.BP_F32, max_batch=max(mb, n)) as net:
+        net.set_weights(theta)
+        net.set_sigmoid(bp.BP_SIGMOID_TABLE)
+        Y = torch.zeros(n, sizes[-1], device="cuda")
+        Xd, Td = dev(X), dev(T)
+        net.forward(Xd, n, Y)
+        net.check()
+        assert normwise(Y.cpu().numpy(), Y_ref) <= TOL
+        sse = torch.zeros(len(e_ref), device="cuda")
+        net.train_epoch(Xd, Td, n, mb, sse)
+        net.check()
+        np.testing.assert_allclose(sse.cpu().numpy(), e_ref, rtol=1e-4, atol=1e-6)
+        assert normwise(net.get_weights() - theta, st.theta - theta) <= 1e-4
+        # back to the logistic: outputs follow the exact oracle again
+        net.set_sigmoid(bp.BP_SIGMOID_LOGISTIC)
+        net.forward(Xd, n, Y)
+        net.check()
+        exact = O.State(sizes, st.theta, lr=0.05, momentum=0.9)
+        assert normwise(Y.cpu().numpy(), O.predict(exact, X)) <= 1e-4
+
+
+def test_table_sigmoid_mode_errors():
+    with bp.Net((4, 3, 2), 0.1, 0.9, bp.BP_F32, max_batch=8) as net:
+        with pytest.raises(bp.BPError) as e:
+            net.set_sigmoid(7)
+        assert e.value.status == bp.BP_EINVAL
+    with bp.Net((256, 128, 64), 0.1, 0.9, bp.BP_BF16, max_batch=128) as net:
+        with pytest.raises(bp.BPError) as e:
+            net.set_sigmoid(bp.BP_SIGMOID_TABLE)
+        assert e.value.status == bp.BP_EINVAL
+
+
 @pytest.mark.parametrize("B", synth.SWEEP_BATCHES)
 def test_batch_sweep_step_matches_oracle(B):
     sizes = (203, 120, 26)
