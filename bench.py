@@ -431,7 +431,7 @@ def run_sweep(args, world, rank, local):
     epochs with the L2 flushed before each.  B <= 4 runs on the one-CTA kernel,
     larger groups on the persistent kernel."""
     import torch
-    from paper_1801_01554_gb300 import bp, synth
+    from paper_1801_01554_gb300 import bp, perf_model, synth
 
     if rank != 0:
         return 0
@@ -464,7 +464,9 @@ def run_sweep(args, world, rank, local):
         net.close()
         t = sorted(ms)[len(ms) // 2] / 1e3
         print(json.dumps({"sweep": "group size", "B": B, "patterns": n, "updates": updates,
-                          "us_per_update": 1e6 * t / updates, "value": W * n / t, "unit": UNIT,
+                          "us_per_update": 1e6 * t / updates,
+                          "model_us_per_update": perf_model.gb300_update_us(B),
+                          "value": W * n / t, "unit": UNIT,
                           "kernel": "one-CTA" if B <= 4 else "persistent cooperative",
                           "dtype": "f32", "data": "synthetic"}), flush=True)
     return 0
