@@ -472,6 +472,54 @@ def run_sweep(args, world, rank, local):
     return 0
 
 
+# ------------------------------------------------------------------ width crossover
+def run_crossover(args, world, rank, local):
+    """fp32 kernels (CUDA cores, weights resident or streamed from L2) against
+    the bf16 GEMM chain (tcgen05 tensor cores) as the hidden layer widens: a
+    208-H-32 net (the NETtalk sizes rounded up to the bf16 path's multiple of
+    8), groups of 512 patterns, one JSON line per H with both times per update."""
+    import torch
+    from paper_1801_01554_gb300 import bp, synth
+
+    if rank != 0:
+        return 0
+    torch.cuda.set_device(local)
+    device = torch.device("cuda", local)
+    B, n = 512, 512 * 32
+    flush = torch.empty(L2_FLUSH_BYTES // 4, dtype=torch.float32, device=device)
+    for H in (64, 128, 256, 512, 1024, 2048, 4096):
+        sizes = (208, H, 32)
+        X, T = synth.gaussian_patterns(n, sizes[0], sizes[-1], 0.1, seed=H)
+        theta = synth.init_normal_fanin(sizes, seed=H)
+        out = {"crossover": "hidden width", "sizes": list(sizes), "B": B, "patterns": n,
+               "connections": connections(sizes)}
+        for name, dt in (("f32", bp.BP_F32), ("bf16", bp.BP_BF16)):
+            Xd = torch.tensor(X, dtype=torch.float32 if dt == bp.BP_F32 else torch.bfloat16,
+                              device=device)
+            Td = torch.tensor(T, dtype=Xd.dtype, device=device)
+            net = bp.Net(sizes, 0.01, 0.9, dt, max_batch=B)
+            net.set_weights(theta)
+            for _ in range(2):
+                net.train_epoch(Xd, Td, n, B)
+            ms = []
+            for k in range(5):
+                flush.fill_(float(k))
+                e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+                e0.record()
+                net.train_epoch(Xd, Td, n, B)
+                e1.record()
+                torch.cuda.synchronize(device)
+                ms.append(e0.elapsed_time(e1))
+            net.check()
+            net.close()
+            t = sorted(ms)[len(ms) // 2] / 1e3
+            out[name + "_us_per_update"] = 1e6 * t / (n // B)
+            out[name + "_cps"] = connections(sizes) * n / t
+        out["faster"] = "bf16" if out["bf16_us_per_update"] < out["f32_us_per_update"] else "f32"
+        print(json.dumps(out), flush=True)
+    return 0
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -485,6 +533,8 @@ def main():
                     help="workload to time (default: the 203-120-26 NETtalk-shaped net)")
     ap.add_argument("--sweep", action="store_true",
                     help="instead of the bench line: CPS against the group size (203-120-26)")
+    ap.add_argument("--crossover", action="store_true",
+                    help="instead of the bench line: fp32 against bf16 as the hidden layer widens")
     args = ap.parse_args()
     if args.warmup < 3 and args.impl == "ours":
         args.warmup = 3
@@ -493,6 +543,8 @@ def main():
         rc = run_reference(args, world, rank)
     elif args.sweep:
         rc = run_sweep(args, world, rank, local)
+    elif args.crossover:
+        rc = run_crossover(args, world, rank, local)
     elif args.workload in ("wide3", "wide4096"):
         rc = run_wide(args, world, rank, local)
     else:
