@@ -193,6 +193,15 @@ def time_oracle(patterns_cap, budget_s, steps=1, warmup=0, min_s=0.0, max_epochs
     return json.loads(r.stdout.strip().splitlines()[-1])
 
 
+# DRAM bytes per pattern of the float32 training kernel on the 203-120-26
+# workload: 15,581,440 bytes (15,299,328 read + 282,112 written) in one ncu
+# capture of a k_train launch over 16,384 patterns with a cold L2
+# (profiles/k_train_nettalk120_launches.md).  The inputs and targets are read
+# once (916 bytes per pattern); everything else stays in L2.  Re-measure after
+# any change to the kernel.
+K_TRAIN_DRAM_BYTES_PER_PATTERN = 15_581_440 / 16_384
+
+
 def connections(sizes):
     return sum((sizes[l - 1] + 1) * sizes[l] for l in range(1, len(sizes)))
 
@@ -340,7 +349,12 @@ def run_ours(args, world, rank, local):
                    "l2": f"flushed ({L2_FLUSH_BYTES >> 20} MB write) before every timed epoch; "
                          "an epoch reads each pattern once"},
         "roofline": {"bound": "alu", "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
-                     "frac": achieved / peak, "traffic": None,
+                     "frac": achieved / peak,
+                     "traffic": K_TRAIN_DRAM_BYTES_PER_PATTERN * n if args.workload == WORKLOAD
+                     else None,
+                     "traffic_basis": "ncu dram__bytes_read.sum + dram__bytes_write.sum of one "
+                                      "k_train launch over 16,384 patterns (cold L2), scaled to "
+                                      "the launch's patterns",
                      "kernel": "k_train (persistent cooperative training kernel)",
                      "peak_basis": f"{num_sms} SMs x {FP32_LANES_PER_SM} FP32 lanes x 2 flop x "
                                    f"{sm_max:.0f} MHz"},
