@@ -194,12 +194,12 @@ def time_oracle(patterns_cap, budget_s, steps=1, warmup=0, min_s=0.0, max_epochs
 
 
 # DRAM bytes per pattern of the float32 training kernel on the 203-120-26
-# workload: 15,581,440 bytes (15,299,328 read + 282,112 written) in one ncu
-# capture of a k_train launch over 16,384 patterns with a cold L2
-# (profiles/k_train_nettalk120_launches.md).  The inputs and targets are read
-# once (916 bytes per pattern); everything else stays in L2.  Re-measure after
-# any change to the kernel.
-K_TRAIN_DRAM_BYTES_PER_PATTERN = 15_581_440 / 16_384
+# workload: 15,537,152 bytes (15,299,584 read + 237,568 written) in one ncu
+# capture of the timed k_train launch of `bench.py --patterns 16384` (16,384
+# patterns after an L2 flush; profiles/k_train_nettalk120_launches.md).  The
+# inputs and targets are read once (916 bytes per pattern); everything else
+# stays in L2.  Re-measure after any change to the kernel.
+K_TRAIN_DRAM_BYTES_PER_PATTERN = 15_537_152 / 16_384
 
 
 def connections(sizes):
@@ -260,7 +260,7 @@ def run_ours(args, world, rank, local):
     torch.cuda.set_device(local)
     device = torch.device("cuda", local)
     w = synth.WORKLOADS[args.workload]
-    sizes, X, T, theta = synth.make_workload(args.workload)
+    sizes, X, T, theta = synth.make_workload(args.workload, patterns=args.patterns)
     n, mb = len(X), w["minibatch"]
     updates = (n + mb - 1) // mb
     W = connections(sizes)
@@ -352,9 +352,9 @@ def run_ours(args, world, rank, local):
                      "frac": achieved / peak,
                      "traffic": K_TRAIN_DRAM_BYTES_PER_PATTERN * n if args.workload == WORKLOAD
                      else None,
-                     "traffic_basis": "ncu dram__bytes_read.sum + dram__bytes_write.sum of one "
-                                      "k_train launch over 16,384 patterns (cold L2), scaled to "
-                                      "the launch's patterns",
+                     "traffic_basis": "ncu dram__bytes_read.sum + dram__bytes_write.sum of the "
+                                      "timed k_train launch of bench.py --patterns 16384 (after "
+                                      "an L2 flush), scaled to the launch's patterns",
                      "kernel": "k_train (persistent cooperative training kernel)",
                      "peak_basis": f"{num_sms} SMs x {FP32_LANES_PER_SM} FP32 lanes x 2 flop x "
                                    f"{sm_max:.0f} MHz"},
@@ -545,6 +545,9 @@ def main():
     ap.add_argument("--workload", default=WORKLOAD,
                     choices=("nettalk60", "nettalk120", "wide3", "wide4096"),
                     help="workload to time (default: the 203-120-26 NETtalk-shaped net)")
+    ap.add_argument("--patterns", type=int, default=None,
+                    help="patterns per epoch (default: the workload's; a smaller epoch of the "
+                         "same net and group size is for profiler captures, not a bench line)")
     ap.add_argument("--sweep", action="store_true",
                     help="instead of the bench line: CPS against the group size (203-120-26)")
     ap.add_argument("--crossover", action="store_true",
