@@ -190,7 +190,10 @@ __device__ __forceinline__ void tmem_ld32(uint32_t taddr, float (&v)[32]) {
     for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
 }
 
-__device__ __forceinline__ float sigmoid_fast(float x) { return 1.0f / (1.0f + __expf(-x)); }
+// Logistic for bf16 outputs: hardware exp2 and the fast reciprocal divide (2 ulp;
+// an IEEE divide here cost a quarter of a training step in the epilogues).
+// For 1 + e^-x beyond 2^126 the quotient is 0, the logistic's value there.
+__device__ __forceinline__ float sigmoid_fast(float x) { return __fdividef(1.0f, 1.0f + __expf(-x)); }
 
 __device__ __forceinline__ float bf16_round(float x) {
     return __bfloat162float(__float2bfloat16_rn(x));
@@ -679,35 +682,56 @@ __global__ void __launch_bounds__(256) k_update_bf16(UpdArgs a) {
         const int tx = threadIdx.x & 31, ty = threadIdx.x >> 5;
         const int rows_w = (u.n_out + 31) / 32;
         if (rb < rows_w) {
-            for (int k = ty; k < 32; k += 8) {
-                const int j = rb * 32 + k, i = cb * 32 + tx;
-                float wv = 0.f;
-                if (j < u.n_out && i < u.n_in) {
-                    const size_t e = (size_t)j * u.n_in + i;
-                    const long long idx = u.woff + (long long)e;
-                    float gsum = 0.f;
-                    if (a.mode != 2) {
-                        for (int s = 0; s < u.splits; ++s)
-                            gsum += u.gpart[(size_t)s * u.n_out * u.n_in + e];
-                    }
-                    if (a.mode == 1) {
-                        a.G[idx] += gsum;
-                        wv = a.theta[idx];
-                    } else if (a.mode == 0) {
-                        if (a.fold_g) {
-                            gsum += a.G[idx];
-                            a.G[idx] = 0.f;
-                        }
-                        const float vel = a.lr_gs * gsum + a.momentum * a.V[idx];
-                        a.V[idx] = vel;
-                        wv = a.theta[idx] + vel;
-                        a.theta[idx] = wv;
-                    } else {
-                        wv = a.theta[idx];
-                    }
-                    if (a.mode != 1) u.wb[e] = __float2bfloat16_rn(wv);
+            // each thread: column i of rows j = rb*32 + ty + 8r (r < 4); every load of
+            // the four rows is issued before any store
+            const int i = cb * 32 + tx;
+            const float* __restrict__ gp = u.gpart;
+            float* __restrict__ th = a.theta;
+            float* __restrict__ vv = a.V;
+            float* __restrict__ gg = a.G;
+            float gsum[4], w0[4], v0[4], gpend[4];
+            bool ok[4];
+            size_t e[4];
+#pragma unroll
+            for (int r = 0; r < 4; ++r) {
+                const int j = rb * 32 + ty + 8 * r;
+                ok[r] = j < u.n_out && i < u.n_in;
+                e[r] = ok[r] ? (size_t)j * u.n_in + i : 0;
+                gsum[r] = 0.f;
+                w0[r] = 0.f;
+                v0[r] = 0.f;
+                gpend[r] = 0.f;
+            }
+#pragma unroll
+            for (int r = 0; r < 4; ++r) {
+                if (!ok[r]) continue;
+                const long long idx = u.woff + (long long)e[r];
+                if (a.mode != 2)
+                    for (int s = 0; s < u.splits; ++s) gsum[r] += __ldcs(gp + (size_t)s * u.n_out * u.n_in + e[r]);
+                w0[r] = th[idx];
+                if (a.mode == 0) {
+                    v0[r] = vv[idx];
+                    if (a.fold_g) gpend[r] = gg[idx];
                 }
-                tileT[k][tx] = __float2bfloat16_rn(wv);
+            }
+#pragma unroll
+            for (int r = 0; r < 4; ++r) {
+                float wv = 0.f;
+                if (ok[r]) {
+                    const long long idx = u.woff + (long long)e[r];
+                    wv = w0[r];
+                    if (a.mode == 1) {
+                        gg[idx] += gsum[r];
+                    } else if (a.mode == 0) {
+                        if (a.fold_g) gg[idx] = 0.f;
+                        const float vel = a.lr_gs * (gsum[r] + gpend[r]) + a.momentum * v0[r];
+                        vv[idx] = vel;
+                        wv += vel;
+                        th[idx] = wv;
+                    }
+                    if (a.mode != 1) u.wb[e[r]] = __float2bfloat16_rn(wv);
+                }
+                tileT[ty + 8 * r][tx] = __float2bfloat16_rn(wv);
             }
             if (a.mode != 1) {
                 __syncthreads();
