@@ -2,6 +2,7 @@
 // float32 (bp_f32.cu) and bfloat16 (bp_bf16.cu) paths.
 #include <cuda_runtime.h>
 
+#include <algorithm>
 #include <cmath>
 #include <cstdarg>
 #include <cstdio>
@@ -78,6 +79,10 @@ struct bp_net {
     void* stage_T = nullptr;
     float* stage_sse = nullptr;
     size_t stage_x_bytes = 0, stage_t_bytes = 0, stage_sse_n = 0;
+    // host-buffer epochs copy piece k + 1 on their own stream while piece k trains
+    cudaStream_t copy_stream = nullptr;
+    cudaEvent_t start_ev = nullptr;
+    cudaEvent_t piece_ev[8] = {};
 };
 
 namespace {
@@ -96,6 +101,10 @@ void free_all(bp_net* net) {
     cudaFree(net->stage_X);
     cudaFree(net->stage_T);
     cudaFree(net->stage_sse);
+    for (cudaEvent_t& e : net->piece_ev)
+        if (e) cudaEventDestroy(e);
+    if (net->start_ev) cudaEventDestroy(net->start_ev);
+    if (net->copy_stream) cudaStreamDestroy(net->copy_stream);
     if (net->bf) bf16_destroy(net->bf);
 }
 
@@ -446,10 +455,41 @@ bp_status bp_train_epoch_host(bp_net* net, const void* h_X, const void* h_T, int
             net->stage_sse_n = ns;
         }
     }
-    BP_CUDA(cudaMemcpyAsync(net->stage_X, h_X, xb, cudaMemcpyHostToDevice, s), "copy X");
-    BP_CUDA(cudaMemcpyAsync(net->stage_T, h_T, tb, cudaMemcpyHostToDevice, s), "copy T");
-    st = run_epoch(net, net->stage_X, net->stage_T, n_patterns, minibatch, net->stage_sse, s);
-    if (st != BP_OK) return st;
+    if (net->copy_stream == nullptr) {
+        BP_CUDA(cudaStreamCreateWithFlags(&net->copy_stream, cudaStreamNonBlocking), "copy stream");
+        BP_CUDA(cudaEventCreateWithFlags(&net->start_ev, cudaEventDisableTiming), "copy events");
+        for (cudaEvent_t& e : net->piece_ev)
+            BP_CUDA(cudaEventCreateWithFlags(&e, cudaEventDisableTiming), "copy events");
+    }
+    // The epoch runs in up to 8 pieces of whole minibatches: the copy of piece
+    // k + 1 (on the net's copy stream) overlaps the training of piece k (on the
+    // caller's stream), which waits for its own piece only.  The staging
+    // buffers may still be read by work queued earlier on the caller's stream.
+    BP_CUDA(cudaEventRecord(net->start_ev, s), "copy events");
+    BP_CUDA(cudaStreamWaitEvent(net->copy_stream, net->start_ev, 0), "copy events");
+    const long long n_steps = (long long)ns;
+    const int pieces = (int)(n_steps < 8 ? n_steps : 8);
+    const long long per = (n_steps + pieces - 1) / pieces;
+    const size_t xrow = (size_t)net->n[0] * elem_size(net);
+    const size_t trow = (size_t)net->n[net->L] * elem_size(net);
+    for (int k = 0; k < pieces; ++k) {
+        const long long step0 = k * per;
+        if (step0 >= n_steps) break;
+        const long long p0 = step0 * minibatch;
+        const long long np = std::min((long long)n_patterns - p0, per * minibatch);
+        char* dx = (char*)net->stage_X + p0 * xrow;
+        char* dt = (char*)net->stage_T + p0 * trow;
+        BP_CUDA(cudaMemcpyAsync(dx, (const char*)h_X + p0 * xrow, np * xrow, cudaMemcpyHostToDevice,
+                                net->copy_stream),
+                "copy X");
+        BP_CUDA(cudaMemcpyAsync(dt, (const char*)h_T + p0 * trow, np * trow, cudaMemcpyHostToDevice,
+                                net->copy_stream),
+                "copy T");
+        BP_CUDA(cudaEventRecord(net->piece_ev[k], net->copy_stream), "copy events");
+        BP_CUDA(cudaStreamWaitEvent(s, net->piece_ev[k], 0), "copy events");
+        st = run_epoch(net, dx, dt, (int)np, minibatch, net->stage_sse + step0, s);
+        if (st != BP_OK) return st;
+    }
     if (h_sse != nullptr)
         BP_CUDA(cudaMemcpyAsync(h_sse, net->stage_sse, ns * sizeof(float), cudaMemcpyDeviceToHost, s),
                 "copy error sums");

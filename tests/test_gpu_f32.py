@@ -292,20 +292,27 @@ def test_checkpoint_resume_is_exact():
         np.testing.assert_array_equal(b.get_weights(), ref)
 
 
-def test_host_buffer_epoch_equals_device_epoch():
-    sizes, n, mb = (203, 120, 26), 3000, 512
+@pytest.mark.parametrize("n,mb", [(3000, 512), (41, 2), (70000, 512)])
+def test_host_buffer_epoch_equals_device_epoch(n, mb):
+    """The host-buffer epoch runs in pieces whose copies overlap training: two
+    epochs in a row give the same bits as two device-buffer epochs."""
+    sizes = (203, 120, 26)
     X, T, theta = problem(sizes, n, seed=17)
     Xh = torch.tensor(X, dtype=torch.float32).pin_memory()
     Th = torch.tensor(T, dtype=torch.float32).pin_memory()
-    sse_h = np.zeros(6, dtype=np.float32)
+    ns = -(-n // mb)
+    sse_h = np.zeros(ns, dtype=np.float32)
     with bp.Net(sizes, 0.05, 0.9, bp.BP_F32, max_batch=mb) as a:
         a.set_weights(theta)
+        a.train_epoch_host(Xh, Th, n, mb, sse_h)
         a.train_epoch_host(Xh, Th, n, mb, sse_h)
         wa = a.get_weights()
     with bp.Net(sizes, 0.05, 0.9, bp.BP_F32, max_batch=mb) as b:
         b.set_weights(theta)
-        sse_d = torch.zeros(6, device="cuda")
-        b.train_epoch(dev(X), dev(T), n, mb, sse_d)
+        sse_d = torch.zeros(ns, device="cuda")
+        Xd, Td = dev(X), dev(T)
+        b.train_epoch(Xd, Td, n, mb, sse_d)
+        b.train_epoch(Xd, Td, n, mb, sse_d)
         np.testing.assert_array_equal(b.get_weights(), wa)
         np.testing.assert_array_equal(sse_d.cpu().numpy(), sse_h)
 
