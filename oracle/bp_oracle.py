@@ -24,7 +24,9 @@ CMU-CS-89-208):
 * the update routine applies the learning rate and momentum to the summed
   change and zeroes the accumulator (Section 6.2.1);
 * optionally, the table-lookup logistic of Section 4.3 (256 points over
-  [-15, 15], linear interpolation, clamped outside) in place of 1/(1+e^-x).
+  [-15, 15], linear interpolation, clamped outside) in place of 1/(1+e^-x);
+* optionally, the fault guard of Section 8: a total weight change outside a
+  reasonable range is set to zero and counted before the update.
 
 Readings taken where the paper is silent (each is listed in the design doc):
 
@@ -192,6 +194,18 @@ def gradients(As, Ds):
     return Gs, gs
 
 
+def guard_changes(g, guard):
+    """The fault guard of Section 8: every total weight change of the group is
+    tested for a reasonable range; one outside it (|g| > guard, or not a
+    number) is set to zero and counted.  guard <= 0 turns the test off.
+    Returns (guarded changes, number zeroed)."""
+    g = np.asarray(g, dtype=np.float64)
+    if guard <= 0:
+        return g, 0
+    bad = ~(np.abs(g) <= guard)
+    return np.where(bad, 0.0, g), int(np.count_nonzero(bad))
+
+
 def momentum_update(w, v, g, lr, momentum, grad_scale=1.0):
     """Update routine of Section 6.2.1 (read as the classic momentum rule):
     v <- lr * grad_scale * g + momentum * v;  w <- w + v.  Returns (w, v)."""
@@ -210,6 +224,8 @@ class State:
     V: np.ndarray = field(default=None)   # previous weight change
     G: np.ndarray = field(default=None)   # pooled change not yet applied
     squash: str = "logistic"              # or "table" (Section 4.3)
+    guard: float = 0.0                    # weight-change range of the fault guard (0: off)
+    faults: int = 0                       # changes the guard has zeroed
 
     def __post_init__(self):
         self.sizes = tuple(int(s) for s in self.sizes)
@@ -238,8 +254,11 @@ def backward_accumulate(state: State, X, T) -> float:
 
 
 def apply_update(state: State) -> None:
-    """Apply and zero the pooled change (Section 6.2.1)."""
-    state.theta, state.V = momentum_update(state.theta, state.V, state.G,
+    """Apply and zero the pooled change (Section 6.2.1), after the fault guard
+    of Section 8 when one is set."""
+    G, n_bad = guard_changes(state.G, state.guard)
+    state.faults += n_bad
+    state.theta, state.V = momentum_update(state.theta, state.V, G,
                                            state.lr, state.momentum, state.grad_scale)
     state.G = np.zeros_like(state.G)
 

@@ -304,3 +304,31 @@ def test_table_squash_changes_a_step_by_at_most_its_error():
     O.train_batch(a, X, T)
     O.train_batch(b, X, T)
     assert np.abs(a.theta - b.theta).max() < 1e-3
+
+
+# ---------------------------------------------------------------- fault guard (Section 8)
+def test_guard_zeroes_and_counts_out_of_range_changes():
+    g = np.array([0.5, -3.0, 2.0, -1.0, np.nan, np.inf, 0.0])
+    out, n = O.guard_changes(g, 1.0)
+    np.testing.assert_array_equal(out, [0.5, 0.0, 0.0, -1.0, 0.0, 0.0, 0.0])
+    assert n == 4
+    same, n0 = O.guard_changes(g[:4], 0.0)          # off
+    np.testing.assert_array_equal(same, g[:4])
+    assert n0 == 0
+
+
+def test_guarded_update_skips_only_the_zeroed_weights():
+    sizes = (4, 3, 2)
+    theta = np.linspace(-0.5, 0.5, O.connections(sizes))
+    X = np.array([[1.0, 0.0, 1.0, 0.0], [0.0, 1.0, 0.0, 1.0]])
+    T = np.array([[1.0, 0.0], [0.0, 1.0]])
+    free = O.State(sizes, theta, lr=0.5, momentum=0.0)
+    O.backward_accumulate(free, X, T)
+    G = free.G.copy()
+    guard = float(np.median(np.abs(G)))
+    st = O.State(sizes, theta, lr=0.5, momentum=0.0, guard=guard)
+    O.train_batch(st, X, T)
+    big = np.abs(G) > guard
+    assert st.faults == int(big.sum()) > 0
+    np.testing.assert_array_equal(st.theta[big], theta[big])
+    np.testing.assert_allclose(st.theta[~big], theta[~big] + 0.5 * G[~big], rtol=0, atol=1e-15)
