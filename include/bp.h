@@ -101,6 +101,19 @@ bp_status bp_set_hparams(bp_net* net, float lr, float momentum, float grad_scale
 enum { BP_SIGMOID_LOGISTIC = 0, BP_SIGMOID_TABLE = 1 };
 bp_status bp_set_sigmoid(bp_net* net, int mode);
 
+/* Fault guard of Section 8: before each update, every total weight change of
+ * the group (the pooled change G, before the learning rate) outside
+ * [-threshold, threshold], or not a number, is set to zero and counted; the
+ * weight then keeps only its momentum term.  threshold = 0 turns the guard off
+ * (the default).  Both dtypes.  Takes effect for work queued after the call.
+ * Errors: BP_EINVAL for a negative or NaN threshold. */
+bp_status bp_set_guard(bp_net* net, float threshold);
+
+/* Number of weight changes the fault guard has zeroed since the net was created
+ * or the count was last reset (reset != 0 resets it after reading).
+ * Synchronises the device.  Errors: BP_EINVAL, BP_ECUDA. */
+bp_status bp_get_faults(bp_net* net, int64_t* count, int reset);
+
 /* Number of float32 values in a parameter vector (W and b of every layer). */
 int64_t bp_num_params(const bp_net* net);
 

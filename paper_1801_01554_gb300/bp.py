@@ -32,6 +32,8 @@ SIGNATURES = {
     "bp_destroy": (None, [_VP]),
     "bp_set_hparams": (_I, [_VP, _F, _F, _F]),
     "bp_set_sigmoid": (_I, [_VP, _I]),
+    "bp_set_guard": (_I, [_VP, _F]),
+    "bp_get_faults": (_I, [_VP, ctypes.POINTER(ctypes.c_int64), _I]),
     "bp_num_params": (ctypes.c_int64, [_VP]),
     "bp_set_weights": (_I, [_VP, _FP]),
     "bp_get_weights": (_I, [_VP, _FP]),
@@ -147,6 +149,16 @@ def bp_set_hparams(h, lr, momentum, grad_scale=1.0):
 
 def bp_set_sigmoid(h, mode):
     _check(load().bp_set_sigmoid(h, int(mode)))
+
+
+def bp_set_guard(h, threshold):
+    _check(load().bp_set_guard(h, float(threshold)))
+
+
+def bp_get_faults(h, reset=False) -> int:
+    c = ctypes.c_int64(0)
+    _check(load().bp_get_faults(h, ctypes.byref(c), 1 if reset else 0))
+    return int(c.value)
 
 
 def bp_num_params(h) -> int:
@@ -272,6 +284,12 @@ class Net:
 
     def set_sigmoid(self, mode):
         bp_set_sigmoid(self.h, mode)
+
+    def set_guard(self, threshold):
+        bp_set_guard(self.h, threshold)
+
+    def get_faults(self, reset=False):
+        return bp_get_faults(self.h, reset)
 
     def set_weights(self, theta):
         bp_set_weights(self.h, theta)

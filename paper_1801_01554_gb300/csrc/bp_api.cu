@@ -202,10 +202,10 @@ bp_status bp_create(const int* sizes, int n_layers, float lr, float momentum, in
         if (e == cudaSuccess) e = cudaMalloc(&net->D, v.d_floats * sizeof(float));
         if (e == cudaSuccess) e = cudaMalloc(&net->sse_part, (size_t)net->num_sms * 4 * sizeof(float));
         if (e == cudaSuccess) e = cudaMalloc(&net->bar, (size_t)bp::kBarWords * sizeof(unsigned));
-        if (e == cudaSuccess) e = cudaMalloc(&net->flags, sizeof(int));
+        if (e == cudaSuccess) e = cudaMalloc(&net->flags, 4 * sizeof(int));
         if (e != cudaSuccess) return bail(cuda_fail(e, "cudaMalloc(scratch)"));
         e = cudaMemset(net->bar, 0, (size_t)bp::kBarWords * sizeof(unsigned));
-        if (e == cudaSuccess) e = cudaMemset(net->flags, 0, sizeof(int));
+        if (e == cudaSuccess) e = cudaMemset(net->flags, 0, 4 * sizeof(int));
         if (e == cudaSuccess) e = cudaMemset(net->A, 0, v.a_floats * sizeof(float));
         if (e == cudaSuccess) e = cudaMemset(net->D, 0, v.d_floats * sizeof(float));
         if (e != cudaSuccess) return bail(cuda_fail(e, "cudaMemset(scratch)"));
@@ -219,6 +219,7 @@ bp_status bp_create(const int* sizes, int n_layers, float lr, float momentum, in
         v.sse_part = net->sse_part;
         v.bar = net->bar;
         v.flags = net->flags;
+        v.faults = reinterpret_cast<unsigned*>(net->flags + 1);
         refresh_view(net);
     } else {
         Bf16Net* b = nullptr;
@@ -226,8 +227,8 @@ bp_status bp_create(const int* sizes, int n_layers, float lr, float momentum, in
                                    net->G, &b);
         if (st != BP_OK) return bail(fail(st, "%s", bf16_last_message()));
         net->bf = b;
-        e = cudaMalloc(&net->flags, sizeof(int));
-        if (e == cudaSuccess) e = cudaMemset(net->flags, 0, sizeof(int));
+        e = cudaMalloc(&net->flags, 4 * sizeof(int));
+        if (e == cudaSuccess) e = cudaMemset(net->flags, 0, 4 * sizeof(int));
         if (e != cudaSuccess) return bail(cuda_fail(e, "cudaMalloc(flags)"));
         bf16_set_flags(b, net->flags);
     }
@@ -260,6 +261,24 @@ bp_status bp_set_sigmoid(bp_net* net, int mode) {
     if (mode == BP_SIGMOID_TABLE && net->dtype != BP_F32)
         return fail(BP_EINVAL, "the table-lookup sigmoid is implemented for float32 nets only");
     net->view.sig_table = mode == BP_SIGMOID_TABLE ? 1 : 0;
+    return BP_OK;
+}
+
+bp_status bp_set_guard(bp_net* net, float threshold) {
+    if (net == nullptr) return fail(BP_EINVAL, "NULL net");
+    if (!(threshold >= 0.f)) return fail(BP_EINVAL, "guard threshold must be >= 0 (0 turns it off)");
+    net->view.guard = threshold;
+    if (net->bf) bf16_set_guard(net->bf, threshold);
+    return BP_OK;
+}
+
+bp_status bp_get_faults(bp_net* net, int64_t* count, int reset) {
+    if (net == nullptr || count == nullptr) return fail(BP_EINVAL, "NULL argument");
+    BP_CUDA(cudaDeviceSynchronize(), "bp_get_faults");
+    unsigned c = 0;
+    BP_CUDA(cudaMemcpy(&c, net->flags + 1, sizeof(unsigned), cudaMemcpyDeviceToHost), "bp_get_faults");
+    *count = (int64_t)c;
+    if (reset) BP_CUDA(cudaMemset(net->flags + 1, 0, sizeof(unsigned)), "bp_get_faults");
     return BP_OK;
 }
 

@@ -658,7 +658,19 @@ struct UpdArgs {
     int n_sse;
     float* sse_out;
     int* flags;
+    float guard;          // > 0: fault guard of Section 8
+    unsigned* faults;     // changes the guard zeroed
 };
+
+// Fault guard of Section 8: a total weight change outside (-guard, guard), or
+// not a number, is set to zero and counted (off while guard <= 0).
+__device__ __forceinline__ float guard_change(const UpdArgs& a, float g) {
+    if (a.guard > 0.f && !(fabsf(g) <= a.guard)) {
+        atomicAdd(a.faults, 1u);
+        return 0.f;
+    }
+    return g;
+}
 
 // Momentum update of Section 6.2.1 over 32x32 weight tiles plus the biases:
 // g = sum of partial changes (+ pending G); v = lr*gs*g + m*v; w += v; then the
@@ -724,7 +736,7 @@ __global__ void __launch_bounds__(256) k_update_bf16(UpdArgs a) {
                         gg[idx] += gsum[r];
                     } else if (a.mode == 0) {
                         if (a.fold_g) gg[idx] = 0.f;
-                        const float vel = a.lr_gs * (gsum[r] + gpend[r]) + a.momentum * v0[r];
+                        const float vel = a.lr_gs * guard_change(a, gsum[r] + gpend[r]) + a.momentum * v0[r];
                         vv[idx] = vel;
                         wv += vel;
                         th[idx] = wv;
@@ -755,7 +767,7 @@ __global__ void __launch_bounds__(256) k_update_bf16(UpdArgs a) {
                         gsum += a.G[idx];
                         a.G[idx] = 0.f;
                     }
-                    const float vel = a.lr_gs * gsum + a.momentum * a.V[idx];
+                    const float vel = a.lr_gs * guard_change(a, gsum) + a.momentum * a.V[idx];
                     a.V[idx] = vel;
                     a.theta[idx] += vel;
                 }
@@ -834,7 +846,8 @@ struct Bf16Net {
     float* theta = nullptr;
     float* V = nullptr;
     float* G = nullptr;
-    int* flags = nullptr;
+    int* flags = nullptr;       // [0] error bits, [1] fault-guard count
+    float guard = 0.f;          // fault guard of Section 8 (0: off)
     long long woff[BP_MAX_SIZES] = {0}, boff[BP_MAX_SIZES] = {0};
     bf16* wb[BP_MAX_SIZES] = {nullptr};     // W_l   [n_l, n_{l-1}]
     bf16* wt[BP_MAX_SIZES] = {nullptr};     // W_l^T [n_{l-1}, n_l]
@@ -1044,6 +1057,8 @@ UpdArgs upd_args(Bf16Net* b, int B, int mode, bool fold, float lr_gs, float mome
     a.n_sse = n_sse;
     a.sse_out = sse_out;
     a.flags = b->flags;
+    a.guard = b->guard;
+    a.faults = reinterpret_cast<unsigned*>(b->flags + 1);
     return a;
 }
 
@@ -1137,6 +1152,7 @@ void bf16_destroy(Bf16Net* b) {
 }
 
 void bf16_set_flags(Bf16Net* b, int* flags) { b->flags = flags; }
+void bf16_set_guard(Bf16Net* b, float guard) { b->guard = guard; }
 
 cudaError_t bf16_refresh_weights(Bf16Net* b, cudaStream_t s) {
     UpdArgs a = upd_args(b, 0, 2, false, 0.f, 0.f, nullptr, 0);

@@ -18,7 +18,8 @@ const char* bf16_last_message();
 bp_status bf16_create(const int* n, int L, int max_batch, int num_sms, float* theta, float* V,
                       float* G, Bf16Net** out);
 void bf16_destroy(Bf16Net* b);
-void bf16_set_flags(Bf16Net* b, int* flags);
+void bf16_set_flags(Bf16Net* b, int* flags);   // flags[0] error bits, flags[1] fault count
+void bf16_set_guard(Bf16Net* b, float guard);  // fault guard of Section 8 (0: off)
 
 // Rewrite the bfloat16 weight copies from the float32 master weights.
 cudaError_t bf16_refresh_weights(Bf16Net* b, cudaStream_t s);

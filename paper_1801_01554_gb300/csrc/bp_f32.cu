@@ -556,6 +556,16 @@ __device__ float pattern_phase(const F32View& v, const PatLayout& q, const float
 }
 
 // ------------------------------------------------------------ weight phase
+// Fault guard of Section 8: a total weight change outside (-guard, guard), or
+// not a number, is set to zero and counted (off while guard <= 0).
+__device__ __forceinline__ float guard_change(const F32View& v, float g) {
+    if (v.guard > 0.f && !(fabsf(g) <= v.guard)) {
+        atomicAdd(v.faults, 1u);
+        return 0.f;
+    }
+    return g;
+}
+
 
 __device__ __forceinline__ void tma_load_2d(float* smem_dst, const CUtensorMap* map, int c0, int c1,
                                             uint64_t* bar) {
@@ -669,6 +679,7 @@ __device__ void weight_phase(const F32View& v, int B, bool fused, bool fold_g, f
                         g += v.G[idx];
                         v.G[idx] = 0.f;
                     }
+                    g = guard_change(v, g);
                     const float vel = v.lr * v.grad_scale * g + v.momentum * v.V[idx];
                     v.V[idx] = vel;
                     v.theta[idx] += vel;
@@ -755,7 +766,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 __global__ void __launch_bounds__(256) k_update(const __grid_constant__ F32View v, long long n) {
     const float a = v.lr * v.grad_scale, m = v.momentum;
     for (long long k = blockIdx.x * 256LL + threadIdx.x; k < n; k += (long long)gridDim.x * 256) {
-        const float vel = a * v.G[k] + m * v.V[k];
+        const float vel = a * guard_change(v, v.G[k]) + m * v.V[k];
         v.V[k] = vel;
         v.theta[k] += vel;
         v.G[k] = 0.f;
@@ -895,6 +906,10 @@ __global__ void __launch_bounds__(kThreads, 1)
                 }
                 float4* wp = reinterpret_cast<float4*>(smem + v.woff[l] + (long long)j * v.kp[l]) + c;
                 float4 w = *wp;
+                g.x = guard_change(v, g.x);
+                g.y = guard_change(v, g.y);
+                g.z = guard_change(v, g.z);
+                g.w = guard_change(v, g.w);
                 float4& u = vel[m];
                 u.x = a_lr * g.x + mom * u.x;
                 u.y = a_lr * g.y + mom * u.y;

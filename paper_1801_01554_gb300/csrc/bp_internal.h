@@ -61,6 +61,8 @@ struct F32View {
     int* flags;           // latched error bits
     float lr, momentum, grad_scale;
     int sig_table;        // 1: table-lookup logistic (Section 4.3) in the forward pass
+    float guard;          // > 0: fault guard of Section 8 (|change| > guard is zeroed)
+    unsigned* faults;     // changes the guard zeroed (flags[1])
     // TMA maps of the weight phase (f32_maps): tm_d[l] over the delta rows of
     // layer l (boxes of 8 columns x 256 patterns), tm_a[l] over the activation
     // rows of layer l (boxes of 32 columns x 256 patterns); zero fill past the

@@ -118,6 +118,7 @@ extern "C" bp_status bp_train_epoch_noalloc(const int* layer_sizes, int n_layers
         return BP_EINVAL;
     }
     v.flags = reinterpret_cast<int*>(base);
+    v.faults = reinterpret_cast<unsigned*>(base + 1);   // the guard stays off here
     v.bar = reinterpret_cast<unsigned*>(base + 4);
     v.sse_part = base + 4 + bar_words;
     float* theta_pad = base + 4 + bar_words + (((long long)sms + 3) & ~3LL);

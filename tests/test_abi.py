@@ -71,4 +71,6 @@ def test_null_handles_are_rejected(lib):
     assert lib.bp_check(None, None) == bp.BP_EINVAL
     assert lib.bp_num_params(None) == 0
     assert lib.bp_set_sigmoid(None, bp.BP_SIGMOID_TABLE) == bp.BP_EINVAL
+    assert lib.bp_set_guard(None, 1.0) == bp.BP_EINVAL
+    assert lib.bp_get_faults(None, None, 0) == bp.BP_EINVAL
     lib.bp_destroy(None)   # NULL-safe

@@ -194,3 +194,27 @@ def test_full_size_workload_sampled(name):
     assert np.any(th != theta.astype(np.float32))
     e_own = float(np.sum((T - y) ** 2))
     assert abs(sse[0].item() - e_own) <= 1e-3 * e_own
+
+
+def test_fault_guard_zeroes_and_counts_on_the_bf16_update():
+    """Section 8's guard on the bf16 update kernel: a threshold below every
+    change zeroes them all (the weights keep their momentum-free values and
+    every nonzero change is counted); a threshold above them all changes nothing."""
+    sizes, B = (64, 128, 32), 256
+    X, T, theta = problem(sizes, B, seed=7)
+    Xd, Td = dev_bf16(X), dev_bf16(T)
+    with bp.Net(sizes, 0.05, 0.9, bp.BP_BF16, max_batch=B) as net:
+        net.set_weights(theta)
+        net.set_guard(1e-30)
+        net.train_batch(Xd, Td, B)
+        net.check()
+        n = net.get_faults(reset=True)
+        assert 0.99 * theta.size <= n <= theta.size
+        np.testing.assert_array_equal(net.get_weights(), theta.astype(np.float32))
+        net.set_guard(1e30)
+        net.train_batch(Xd, Td, B)
+        net.check()
+        assert net.get_faults() == 0
+        st = O.State(sizes, theta, lr=0.05, momentum=0.9)
+        O.train_batch(st, X, T)
+        assert normwise(net.get_weights() - theta, st.theta - theta) <= TOL

@@ -205,6 +205,68 @@ def test_table_sigmoid_mode_errors():
         assert e.value.status == bp.BP_EINVAL
 
 
+def _gap_threshold(G):
+    """A guard threshold between two consecutive |G| values near the median,
+    far (relative to fp32 rounding) from both, so that both sides zero the same
+    changes."""
+    a = np.sort(np.abs(G[G != 0]))
+    mid = len(a) // 2
+    for k in range(mid, len(a) - 1):
+        if a[k + 1] > a[k] * (1 + 1e-3):
+            return 0.5 * (a[k] + a[k + 1])
+    raise AssertionError("no gap")
+
+
+@pytest.mark.parametrize("B", [512, 2])
+def test_fault_guard_matches_oracle(B):
+    """Section 8's guard on the persistent (B = 512) and one-CTA (B = 2) kernels:
+    the same changes are zeroed and counted, the other weights update as usual."""
+    sizes = (203, 120, 26)
+    X, T, theta = problem(sizes, B, seed=41)
+    probe = O.State(sizes, theta, lr=0.05, momentum=0.9)
+    O.backward_accumulate(probe, X, T)
+    guard = _gap_threshold(probe.G)
+    st = O.State(sizes, theta, lr=0.05, momentum=0.9, guard=guard)
+    O.train_batch(st, X, T)
+    with bp.Net(sizes, 0.05, 0.9, bp.BP_F32, max_batch=B) as net:
+        net.set_weights(theta)
+        net.set_guard(guard)
+        net.train_batch(dev(X), dev(T), B)
+        net.check()
+        assert net.get_faults(reset=True) == st.faults > 0
+        assert net.get_faults() == 0
+        assert normwise(net.get_weights() - theta, st.theta - theta) <= TOL
+
+
+def test_fault_guard_on_backward_then_update_and_off_by_default():
+    sizes, B = (64, 33, 17, 9), 300
+    X, T, theta = problem(sizes, B, seed=42)
+    probe = O.State(sizes, theta, lr=0.1, momentum=0.9)
+    O.backward_accumulate(probe, X, T)
+    guard = _gap_threshold(probe.G)
+    st = O.State(sizes, theta, lr=0.1, momentum=0.9, guard=guard)
+    O.backward_accumulate(st, X, T)
+    O.apply_update(st)
+    with bp.Net(sizes, 0.1, 0.9, bp.BP_F32, max_batch=B) as net:
+        net.set_weights(theta)
+        Xd, Td = dev(X), dev(T)
+        net.forward(Xd, B)
+        net.backward(Td, B)
+        net.set_guard(guard)
+        net.update()
+        net.check()
+        assert net.get_faults() == st.faults > 0
+        assert normwise(net.get_weights() - theta, st.theta - theta) <= TOL
+        # off again: a step zeroes nothing
+        net.set_guard(0.0)
+        net.get_faults(reset=True)
+        net.train_batch(Xd, Td, B)
+        net.check()
+        assert net.get_faults() == 0
+        with pytest.raises(bp.BPError):
+            net.set_guard(-1.0)
+
+
 @pytest.mark.parametrize("B", synth.SWEEP_BATCHES)
 def test_batch_sweep_step_matches_oracle(B):
     sizes = (203, 120, 26)
