@@ -114,6 +114,25 @@ bp_status bp_set_guard(bp_net* net, float threshold);
  * Synchronises the device.  Errors: BP_EINVAL, BP_ECUDA. */
 bp_status bp_get_faults(bp_net* net, int64_t* count, int reset);
 
+/* Diagnostic mode (Section 8): every CTA of one launch, one per SM, runs the
+ * forward pass and the summed squared error of the same `batch` patterns
+ * (device d_X [batch, n_0], d_T [batch, n_L]) with the net's weights, without
+ * exchanging anything with the others, as each GF11 processor ran the same
+ * training set alone.  The per-CTA error sums go to h_sse and the SM each CTA
+ * ran on to h_sm (host arrays of `capacity` >= the SM count; either may be
+ * NULL); *n_ctas receives the number of CTAs and *n_agree how many produced the
+ * most common error sum, bit for bit (a healthy GPU: all of them).  Leaves the
+ * weights alone.  Synchronous.  Float32 nets only.
+ * Errors: BP_EINVAL (NULL pointers, a BP_BF16 net, capacity too small, batch
+ * out of range), BP_ECUDA. */
+bp_status bp_diagnose(bp_net* net, const void* d_X, const void* d_T, int batch, float* h_sse,
+                      int* h_sm, int capacity, int* n_ctas, int* n_agree);
+
+/* The host's vote of the diagnostic mode: the value that most of values[0, n)
+ * equal bit for bit goes to *mode (may be NULL; ties: the earliest such value)
+ * and its count to *n_agree.  Host only.  Errors: BP_EINVAL. */
+bp_status bp_vote(const float* values, int n, float* mode, int* n_agree);
+
 /* Number of float32 values in a parameter vector (W and b of every layer). */
 int64_t bp_num_params(const bp_net* net);
 

@@ -34,6 +34,9 @@ SIGNATURES = {
     "bp_set_sigmoid": (_I, [_VP, _I]),
     "bp_set_guard": (_I, [_VP, _F]),
     "bp_get_faults": (_I, [_VP, ctypes.POINTER(ctypes.c_int64), _I]),
+    "bp_diagnose": (_I, [_VP, _VP, _VP, _I, _FP, ctypes.POINTER(_I), _I, ctypes.POINTER(_I),
+                         ctypes.POINTER(_I)]),
+    "bp_vote": (_I, [_FP, _I, _FP, ctypes.POINTER(_I)]),
     "bp_num_params": (ctypes.c_int64, [_VP]),
     "bp_set_weights": (_I, [_VP, _FP]),
     "bp_get_weights": (_I, [_VP, _FP]),
@@ -159,6 +162,27 @@ def bp_get_faults(h, reset=False) -> int:
     c = ctypes.c_int64(0)
     _check(load().bp_get_faults(h, ctypes.byref(c), 1 if reset else 0))
     return int(c.value)
+
+
+def bp_diagnose(h, X, T, batch, capacity=1024):
+    """Diagnostic mode: (per-CTA error sums, SM ids, number agreeing with the vote)."""
+    sse = np.zeros(capacity, dtype=np.float32)
+    sm = np.zeros(capacity, dtype=np.int32)
+    n = ctypes.c_int(0)
+    agree = ctypes.c_int(0)
+    _check(load().bp_diagnose(h, _dptr(X), _dptr(T), int(batch), sse.ctypes.data_as(_FP),
+                              sm.ctypes.data_as(ctypes.POINTER(_I)), capacity, ctypes.byref(n),
+                              ctypes.byref(agree)))
+    return sse[:n.value], sm[:n.value], agree.value
+
+
+def bp_vote(values):
+    """(the value most entries equal bit for bit, how many equal it)."""
+    a = np.ascontiguousarray(values, dtype=np.float32)
+    mode = ctypes.c_float(0.0)
+    agree = ctypes.c_int(0)
+    _check(load().bp_vote(a.ctypes.data_as(_FP), int(a.size), ctypes.byref(mode), ctypes.byref(agree)))
+    return float(mode.value), agree.value
 
 
 def bp_num_params(h) -> int:
@@ -290,6 +314,9 @@ class Net:
 
     def get_faults(self, reset=False):
         return bp_get_faults(self.h, reset)
+
+    def diagnose(self, X, T, batch):
+        return bp_diagnose(self.h, X, T, batch)
 
     def set_weights(self, theta):
         bp_set_weights(self.h, theta)

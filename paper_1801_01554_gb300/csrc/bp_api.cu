@@ -83,6 +83,7 @@ struct bp_net {
     cudaStream_t copy_stream = nullptr;
     cudaEvent_t start_ev = nullptr;
     cudaEvent_t piece_ev[8] = {};
+    int* diag_sm = nullptr;   // bp_diagnose: SM of each CTA
 };
 
 namespace {
@@ -105,6 +106,7 @@ void free_all(bp_net* net) {
         if (e) cudaEventDestroy(e);
     if (net->start_ev) cudaEventDestroy(net->start_ev);
     if (net->copy_stream) cudaStreamDestroy(net->copy_stream);
+    cudaFree(net->diag_sm);
     if (net->bf) bf16_destroy(net->bf);
 }
 
@@ -280,6 +282,47 @@ bp_status bp_get_faults(bp_net* net, int64_t* count, int reset) {
     *count = (int64_t)c;
     if (reset) BP_CUDA(cudaMemset(net->flags + 1, 0, sizeof(unsigned)), "bp_get_faults");
     return BP_OK;
+}
+
+bp_status bp_vote(const float* values, int n, float* mode, int* n_agree) {
+    if (values == nullptr || n < 1 || n_agree == nullptr) return fail(BP_EINVAL, "bad argument");
+    // the value most CTAs produced, bit for bit (ties: the first such value)
+    int best = 0, best_count = 0;
+    for (int i = 0; i < n; ++i) {
+        int c = 0;
+        for (int k = 0; k < n; ++k) c += std::memcmp(&values[i], &values[k], sizeof(float)) == 0;
+        if (c > best_count) {
+            best = i;
+            best_count = c;
+        }
+    }
+    if (mode != nullptr) *mode = values[best];
+    *n_agree = best_count;
+    return BP_OK;
+}
+
+bp_status bp_diagnose(bp_net* net, const void* d_X, const void* d_T, int batch, float* h_sse,
+                      int* h_sm, int capacity, int* n_ctas, int* n_agree) {
+    if (net == nullptr || d_X == nullptr || d_T == nullptr || n_ctas == nullptr || n_agree == nullptr)
+        return fail(BP_EINVAL, "NULL argument");
+    if (net->dtype != BP_F32) return fail(BP_EINVAL, "the diagnostic mode is implemented for float32 nets");
+    bp_status st = check_batch(net, batch);
+    if (st != BP_OK) return st;
+    const int n = net->num_sms;
+    if ((h_sse != nullptr || h_sm != nullptr) && capacity < n)
+        return fail(BP_EINVAL, "capacity %d is below the %d CTAs of the launch", capacity, n);
+    if (net->diag_sm == nullptr) BP_CUDA(cudaMalloc(&net->diag_sm, n * sizeof(int)), "cudaMalloc(diagnose)");
+    BP_CUDA(f32_diagnose(net->view, (const float*)d_X, (const float*)d_T, batch, net->sse_part,
+                         net->diag_sm, n, 0),
+            "bp_diagnose");
+    std::vector<float> sse(n);
+    std::vector<int> sm(n);
+    BP_CUDA(cudaMemcpy(sse.data(), net->sse_part, n * sizeof(float), cudaMemcpyDeviceToHost), "bp_diagnose");
+    BP_CUDA(cudaMemcpy(sm.data(), net->diag_sm, n * sizeof(int), cudaMemcpyDeviceToHost), "bp_diagnose");
+    if (h_sse != nullptr) std::memcpy(h_sse, sse.data(), n * sizeof(float));
+    if (h_sm != nullptr) std::memcpy(h_sm, sm.data(), n * sizeof(int));
+    *n_ctas = n;
+    return bp_vote(sse.data(), n, nullptr, n_agree);
 }
 
 int64_t bp_num_params(const bp_net* net) { return net ? (int64_t)net->P : 0; }

@@ -25,6 +25,7 @@
 // barrier is bounded and latches kFlagTimeout instead of hanging.
 #include <cuda_runtime.h>
 
+#include <algorithm>
 #include <cmath>
 #include <cstdio>
 
@@ -470,20 +471,21 @@ __device__ __forceinline__ void rows_to_global(float* dst, const float* src, int
 //       loads overlap
 //   to_scratch: write the activation and delta rows to scratch (A, D)
 //   rows_issued: the first pass's rows were already issued (load_rows)
+//   whole: this CTA takes all B patterns (diagnostic mode) instead of its share
 template <int PG>
 __device__ float pattern_phase(const F32View& v, const PatLayout& q, const float* Wb,
                                const float* __restrict__ X, const float* __restrict__ T, int B,
                                bool do_fwd, bool do_bwd, float* __restrict__ Y, float* smem,
                                const WeightCopy* wc = nullptr, bool to_scratch = true,
-                               bool rows_issued = false) {
+                               bool rows_issued = false, bool whole = false) {
     constexpr int TP = kThreads / PG;
     const int L = v.L;
     const int tid = threadIdx.x;
     const int pr = tid / TP, c0 = tid % TP;   // row-loop split
     const int nL = v.n[L];
     float sse = 0.f;
-    const int q_lo = (int)((long long)B * blockIdx.x / gridDim.x);
-    const int q_hi = (int)((long long)B * (blockIdx.x + 1) / gridDim.x);
+    const int q_lo = whole ? 0 : (int)((long long)B * blockIdx.x / gridDim.x);
+    const int q_hi = whole ? B : (int)((long long)B * (blockIdx.x + 1) / gridDim.x);
     for (int p0 = q_lo; p0 < q_hi; p0 += PG) {
         const int np = min(PG, q_hi - p0);
         if (!(rows_issued && p0 == q_lo))
@@ -753,6 +755,35 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (threadIdx.x == 0) v.sse_part[blockIdx.x] = e;
 }
 
+// Diagnostic mode (Section 8): every CTA runs the forward pass and the error of
+// all B patterns with the same weights, independently of the others, and
+// reports its summed squared error and the SM it ran on.
+template <int PG, bool WS>
+__global__ void __launch_bounds__(kThreads, 1)
+    k_diagnose(const __grid_constant__ F32View v, const PatLayout q, const float* X, const float* T,
+               int B, float* sse_out, int* sm_out) {
+    extern __shared__ __align__(128) float smem[];
+    __shared__ __align__(8) uint64_t s_bar;
+    unsigned phase = 0;
+    sigmoid_table_init(v);
+    mbar_init1(&s_bar);
+    float e;
+    if (WS) {
+        stage_weights(v.theta, v.P, smem, &s_bar, phase, v.flags);
+        e = pattern_phase<PG>(v, q, smem, X, T, B, true, true, nullptr, pattern_base<true>(v, smem),
+                              nullptr, false, false, true);
+    } else {
+        e = pattern_phase<PG>(v, q, v.theta, X, T, B, true, true, nullptr, pattern_base<false>(v, smem),
+                              nullptr, false, false, true);
+    }
+    if (threadIdx.x == 0) {
+        unsigned sm;
+        asm volatile("mov.u32 %0, %%smid;" : "=r"(sm));
+        sse_out[blockIdx.x] = e;
+        sm_out[blockIdx.x] = (int)sm;
+    }
+}
+
 __global__ void __launch_bounds__(kThreads, 1)
     k_accumulate(const __grid_constant__ F32View v, int B, int nparts, float* sse_out) {
     extern __shared__ __align__(128) float smem[];
@@ -970,6 +1001,9 @@ __global__ void __launch_bounds__(256) k_unpad(const __grid_constant__ F32View v
 template <int PG, bool WS>
 cudaError_t set_smem_attr_ws(size_t bytes) {
     cudaError_t e;
+    if ((e = cudaFuncSetAttribute(k_diagnose<PG, WS>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                  (int)bytes)) != cudaSuccess)
+        return e;
     if ((e = cudaFuncSetAttribute(k_forward<PG, WS>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                   (int)bytes)) != cudaSuccess)
         return e;
@@ -1277,6 +1311,25 @@ cudaError_t f32_train_small(const F32View& v, const float* X, const float* T, in
         default: if (big) BP_SMALL(4, 16); else BP_SMALL(4, 4); break;
     }
 #undef BP_SMALL
+    return cudaGetLastError();
+}
+
+// ------------------------------------------------------------ diagnostic mode
+cudaError_t f32_diagnose(const F32View& v, const float* X, const float* T, int batch, float* d_sse,
+                         int* d_sm, int num_sms, cudaStream_t s) {
+    // every CTA takes all `batch` patterns: plan as if each had that many
+    const F32Plan plan = f32_plan(v, (int)std::min<long long>((long long)batch * num_sms, 1 << 30), num_sms);
+#define BP_DIAG(PG)                                                                          \
+    (plan.w_in_smem                                                                          \
+         ? (k_diagnose<PG, true><<<num_sms, kThreads, plan.smem, s>>>(v, plan.q, X, T, batch, d_sse, d_sm)) \
+         : (k_diagnose<PG, false><<<num_sms, kThreads, plan.smem, s>>>(v, plan.q, X, T, batch, d_sse, d_sm)))
+    switch (plan.pg) {
+        case 1: BP_DIAG(1); break;
+        case 2: BP_DIAG(2); break;
+        case 4: BP_DIAG(4); break;
+        default: BP_DIAG(8); break;
+    }
+#undef BP_DIAG
     return cudaGetLastError();
 }
 

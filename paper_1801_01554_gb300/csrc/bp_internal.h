@@ -132,6 +132,11 @@ bool f32_small_ok(const F32View& v, int minibatch);
 cudaError_t f32_train_small(const F32View& v, const float* X, const float* T, int n_patterns,
                             int minibatch, int n_steps, float* sse_out, cudaStream_t s);
 
+// Diagnostic mode (Section 8): num_sms CTAs each run the forward pass and error
+// of all `batch` patterns; per-CTA error sums to d_sse, SM ids to d_sm.
+cudaError_t f32_diagnose(const F32View& v, const float* X, const float* T, int batch, float* d_sse,
+                         int* d_sm, int num_sms, cudaStream_t s);
+
 // Message returned by bp_last_error() on the calling thread (bp_api.cu).
 void set_error_message(const char* msg);
 

@@ -267,6 +267,24 @@ def test_fault_guard_on_backward_then_update_and_off_by_default():
             net.set_guard(-1.0)
 
 
+@pytest.mark.parametrize("sizes,B", [((203, 120, 26), 64), ((64, 33, 17, 9), 37)])
+def test_diagnostic_mode_every_sm_agrees(sizes, B):
+    """Section 8's diagnostic mode: every CTA (one per SM) computes the error of
+    the same patterns alone; on a healthy GPU they agree bit for bit, with the
+    oracle's error sum, and the weights are left alone."""
+    X, T, theta = problem(sizes, B, seed=51)
+    st = O.State(sizes, theta, lr=0.05, momentum=0.9)
+    e_ref = O.sse(O.predict(st, X), T)
+    with bp.Net(sizes, 0.05, 0.9, bp.BP_F32, max_batch=B) as net:
+        net.set_weights(theta)
+        sse, sm, agree = net.diagnose(dev(X), dev(T), B)
+        n_sm = torch.cuda.get_device_properties(0).multi_processor_count
+        assert len(sse) == n_sm and agree == n_sm
+        assert np.all(sse == sse[0]) and abs(float(sse[0]) - e_ref) <= TOL * e_ref
+        assert np.all((sm >= 0) & (sm < n_sm))
+        np.testing.assert_array_equal(net.get_weights(), theta.astype(np.float32))
+
+
 @pytest.mark.parametrize("B", synth.SWEEP_BATCHES)
 def test_batch_sweep_step_matches_oracle(B):
     sizes = (203, 120, 26)
