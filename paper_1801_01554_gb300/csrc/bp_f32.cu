@@ -355,92 +355,23 @@ __device__ void forward_layer(const float* W, int kp, int n_out, const float* s_
     }
 }
 
-// PG consecutive floats (16-byte aligned when PG >= 4) into registers.
-template <int PG>
-__device__ __forceinline__ void load_pg(const float* p, float (&d)[PG]) {
-    if constexpr (PG >= 4) {
-#pragma unroll
-        for (int k = 0; k < PG; k += 4) {
-            const float4 x = *reinterpret_cast<const float4*>(p + k);
-            d[k] = x.x;
-            d[k + 1] = x.y;
-            d[k + 2] = x.z;
-            d[k + 3] = x.w;
-        }
-    } else if constexpr (PG == 2) {
-        const float2 x = *reinterpret_cast<const float2*>(p);
-        d[0] = x.x;
-        d[1] = x.y;
-    } else {
-        d[0] = p[0];
-    }
-}
-
 // Hidden deltas of layer l for PG patterns: d_l[p][i] = (sum_j W_{l+1}[j][i]
-// d_{l+1}[p][j]) a_l[p][i] (1 - a_l[p][i]).  dnt holds d_{l+1} pattern-minor
-// ([nn][PG]) so that one vector load gives a column's PG deltas.  Units go to
-// threads; when there are fewer than kThreads units, the sum over j is split
-// over JS interleaved slices whose partials meet in shared memory in a fixed
-// order.  Writes d_l as rows (dl, pitch dpl) and, if dlt is not null,
-// pattern-minor (dlt).
+// d_{l+1}[p][j]) a_l[p][i] (1 - a_l[p][i]), one thread per (pattern, unit)
+// summing over the next layer's units in order.  dnt holds d_{l+1}
+// pattern-minor ([nn][PG]).  Writes d_l as rows (dl, pitch dpl) and, if dlt is
+// not null, pattern-minor (dlt).
 template <int PG>
 __device__ void hidden_delta(const float* Wn, int kpn, int n, int nn, const float* dnt,
-                             const float* al, int apl, float* dl, int dpl, float* dlt, float* red) {
-    const int tid = threadIdx.x;
-    const int NI = (n + 31) & ~31;
-    const int JS = NI < kThreads ? kThreads / NI : 1;
-    if (JS > 1) {
-        const int sl = tid / NI, i = tid - sl * NI;
-        float acc[PG];
-#pragma unroll
-        for (int p = 0; p < PG; ++p) acc[p] = 0.f;
-        if (sl < JS && i < n) {
-#pragma unroll 2
-            for (int j = sl; j < nn; j += JS) {
-                const float w = Wn[(size_t)j * kpn + i];
-                float d[PG];
-                load_pg<PG>(dnt + j * PG, d);
-#pragma unroll
-                for (int p = 0; p < PG; ++p) acc[p] = fmaf(d[p], w, acc[p]);
-            }
-        }
-        if (sl < JS) {
-#pragma unroll
-            for (int p = 0; p < PG; ++p) red[(sl * PG + p) * NI + i] = acc[p];
-        }
-        __syncthreads();
-        if (tid < n) {
-#pragma unroll
-            for (int p = 0; p < PG; ++p) {
-                float g = 0.f;
-                for (int k = 0; k < JS; ++k) g += red[(k * PG + p) * NI + tid];
-                const float a = al[p * apl + tid];
-                const float d = g * a * (1.f - a);
-                dl[p * dpl + tid] = d;
-                if (dlt != nullptr) dlt[tid * PG + p] = d;
-            }
-        }
-    } else {
-        for (int i = tid; i < n; i += kThreads) {
-            float acc[PG];
-#pragma unroll
-            for (int p = 0; p < PG; ++p) acc[p] = 0.f;
-#pragma unroll 2
-            for (int j = 0; j < nn; ++j) {
-                const float w = Wn[(size_t)j * kpn + i];
-                float d[PG];
-                load_pg<PG>(dnt + j * PG, d);
-#pragma unroll
-                for (int p = 0; p < PG; ++p) acc[p] = fmaf(d[p], w, acc[p]);
-            }
-#pragma unroll
-            for (int p = 0; p < PG; ++p) {
-                const float a = al[p * apl + i];
-                const float d = acc[p] * a * (1.f - a);
-                dl[p * dpl + i] = d;
-                if (dlt != nullptr) dlt[i * PG + p] = d;
-            }
-        }
+                             const float* al, int apl, float* dl, int dpl, float* dlt) {
+    for (int e = threadIdx.x; e < PG * n; e += kThreads) {
+        const int p = e / n, i = e - p * n;
+        float acc = 0.f;
+#pragma unroll 4
+        for (int j = 0; j < nn; ++j) acc = fmaf(dnt[j * PG + p], Wn[(size_t)j * kpn + i], acc);
+        const float a = al[p * apl + i];
+        const float d = acc * a * (1.f - a);
+        dl[p * dpl + i] = d;
+        if (dlt != nullptr) dlt[i * PG + p] = d;
     }
 }
 
@@ -542,7 +473,7 @@ __device__ float pattern_phase(const F32View& v, const PatLayout& q, const float
             for (int l = L - 1; l >= 1; --l) {
                 hidden_delta<PG>(Wb + v.woff[l + 1], v.kp[l + 1], v.n[l], v.n[l + 1], smem + q.sdt[l + 1],
                                  smem + q.sa[l], v.apitch[l], smem + q.sd[l], v.dpitch[l],
-                                 l >= 2 ? smem + q.sdt[l] : nullptr, smem + q.red);
+                                 l >= 2 ? smem + q.sdt[l] : nullptr);
                 __syncthreads();
             }
             for (int l = 1; l <= L && to_scratch; ++l)
@@ -566,6 +497,13 @@ __device__ __forceinline__ float guard_change(const F32View& v, float g) {
         return 0.f;
     }
     return g;
+}
+
+// The same test without an atomic per change: zeroes and counts into n_bad.
+__device__ __forceinline__ float guard_count(float guard, float g, unsigned& n_bad) {
+    const bool bad = guard > 0.f && !(fabsf(g) <= guard);
+    n_bad += bad ? 1u : 0u;
+    return bad ? 0.f : g;
 }
 
 
@@ -865,7 +803,9 @@ struct SmallPlan {
     int m0[BP_MAX_SIZES + 1];
 };
 
-template <int PG, int NV4>
+// GUARD: the fault guard is on (a separate instantiation, so that the update
+// loop carries no test when it is off).
+template <int PG, int NV4, bool GUARD>
 __global__ void __launch_bounds__(kThreads, 1)
     k_train_small(const __grid_constant__ F32View v, const PatLayout q, const SmallPlan sp,
                   const float* X, const float* T, int n_patterns, int minibatch, int n_steps,
@@ -891,7 +831,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                       : make_float4(0.f, 0.f, 0.f, 0.f);
     }
     stage_weights(v.theta, v.P, smem, &s_bar, phase, v.flags);
-    const float a_lr = v.lr * v.grad_scale, mom = v.momentum;
+    const float a_lr = v.lr * v.grad_scale, mom = v.momentum, guard = v.guard;
     if (n_steps > 0)
         load_rows<PG>(v, q, X, T, 0, (int)min((long long)minibatch, (long long)n_patterns), pat[0]);
     for (int s = 0; s < n_steps; ++s) {
@@ -911,6 +851,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         // momentum update of every weight from this group's deltas and inputs
         int l = 0, K4 = 1, c = 0, j0 = 0, R = 1;
+        unsigned n_bad = 0;
         float4 a[PG];
 #pragma unroll
         for (int m = 0; m < NV4; ++m) {
@@ -937,10 +878,12 @@ __global__ void __launch_bounds__(kThreads, 1)
                 }
                 float4* wp = reinterpret_cast<float4*>(smem + v.woff[l] + (long long)j * v.kp[l]) + c;
                 float4 w = *wp;
-                g.x = guard_change(v, g.x);
-                g.y = guard_change(v, g.y);
-                g.z = guard_change(v, g.z);
-                g.w = guard_change(v, g.w);
+                if (GUARD) {
+                    g.x = guard_count(guard, g.x, n_bad);
+                    g.y = guard_count(guard, g.y, n_bad);
+                    g.z = guard_count(guard, g.z, n_bad);
+                    g.w = guard_count(guard, g.w, n_bad);
+                }
                 float4& u = vel[m];
                 u.x = a_lr * g.x + mom * u.x;
                 u.y = a_lr * g.y + mom * u.y;
@@ -953,6 +896,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 *wp = w;
             }
         }
+        if (GUARD && n_bad != 0) atomicAdd(v.faults, n_bad);
         __syncthreads();
     }
     // weights and weight changes back to global memory
@@ -1076,8 +1020,6 @@ static PatLayout pat_layout(const int* n, int L, int pg) {
     for (int l = 2; l <= L; ++l) { q.sdt[l] = off; off += (pg * n[l] + 3) & ~3; }
     q.st = off;
     off += (pg * n[L] + 3) & ~3;
-    q.red = off;
-    off += kThreads * pg;
     q.total = off;
     return q;
 }
@@ -1144,13 +1086,20 @@ cudaError_t f32_maps(F32View& v) {
     return cudaSuccess;
 }
 
+template <int PG, bool GUARD>
+cudaError_t set_small_attr_g(size_t bytes) {
+    cudaError_t e = cudaFuncSetAttribute(k_train_small<PG, 4, GUARD>,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize, (int)bytes);
+    if (e != cudaSuccess) return e;
+    return cudaFuncSetAttribute(k_train_small<PG, 16, GUARD>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                (int)bytes);
+}
+
 template <int PG>
 cudaError_t set_small_attr(size_t bytes) {
-    cudaError_t e = cudaFuncSetAttribute(k_train_small<PG, 4>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         (int)bytes);
+    cudaError_t e = set_small_attr_g<PG, false>(bytes);
     if (e != cudaSuccess) return e;
-    return cudaFuncSetAttribute(k_train_small<PG, 16>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                (int)bytes);
+    return set_small_attr_g<PG, true>(bytes);
 }
 
 cudaError_t f32_setup(int device) {
@@ -1302,9 +1251,12 @@ cudaError_t f32_train_small(const F32View& v, const float* X, const float* T, in
     const SmallPlan sp = small_plan(v);
     const size_t bytes = ((size_t)v.wsm + 2 * (size_t)q.total) * sizeof(float);
     const bool big = sp.m0[v.L + 1] > 4;
-#define BP_SMALL(PG, NV)                                                                        \
-    k_train_small<PG, NV><<<1, kThreads, bytes, s>>>(v, q, sp, X, T, n_patterns, minibatch, n_steps, \
-                                                     sse_out)
+#define BP_SMALL(PG, NV)                                                                           \
+    (v.guard > 0.f                                                                                  \
+         ? k_train_small<PG, NV, true><<<1, kThreads, bytes, s>>>(v, q, sp, X, T, n_patterns, minibatch, \
+                                                                  n_steps, sse_out)                 \
+         : k_train_small<PG, NV, false><<<1, kThreads, bytes, s>>>(v, q, sp, X, T, n_patterns,          \
+                                                                   minibatch, n_steps, sse_out))
     switch (pg) {
         case 1: if (big) BP_SMALL(1, 16); else BP_SMALL(1, 4); break;
         case 2: if (big) BP_SMALL(2, 16); else BP_SMALL(2, 4); break;

@@ -76,14 +76,12 @@ struct F32View {
 // patterns, computed on the host: activation rows sa[l] ([PG][apitch_l],
 // l = 0..L), delta rows sd[l] ([PG][dpitch_l], l = 1..L), the same deltas
 // pattern-minor sdt[l] ([n_l][PG], l = 2..L, read by the hidden deltas below
-// them), target rows st ([PG][n_L]) and hidden-delta partial sums red
-// (kThreads * PG floats); `total` floats in all.
+// them) and target rows st ([PG][n_L]); `total` floats in all.
 struct PatLayout {
     int sa[BP_MAX_SIZES];
     int sd[BP_MAX_SIZES];
     int sdt[BP_MAX_SIZES];
     int st;
-    int red;
     int total;
 };
 
