@@ -218,3 +218,24 @@ def test_fault_guard_zeroes_and_counts_on_the_bf16_update():
         st = O.State(sizes, theta, lr=0.05, momentum=0.9)
         O.train_batch(st, X, T)
         assert normwise(net.get_weights() - theta, st.theta - theta) <= TOL
+
+
+def test_deepest_net_the_boundary_allows():
+    """BP_MAX_SIZES layer sizes (8 weight layers): outputs and one update's
+    weight change, held to the same 2e-2 as every bf16 step."""
+    sizes = (8, 16, 8, 24, 8, 16, 8, 16, 8)
+    assert len(sizes) == bp.BP_MAX_SIZES
+    B = 40
+    X, T, theta = problem(sizes, B, seed=9)
+    st = O.State(sizes, theta, lr=0.1, momentum=0.9)
+    Y_ref = O.predict(st, X)
+    O.train_batch(st, X, T)
+    with bp.Net(sizes, 0.1, 0.9, bp.BP_BF16, max_batch=B) as net:
+        net.set_weights(theta)
+        Xd, Td = dev_bf16(X), dev_bf16(T)
+        Y = torch.zeros(B, sizes[-1], dtype=torch.bfloat16, device="cuda")
+        net.forward(Xd, B, Y)
+        net.train_batch(Xd, Td, B)
+        net.check()
+        assert normwise(Y.float().cpu().numpy(), Y_ref) <= TOL
+        assert normwise(net.get_weights() - theta, st.theta - theta) <= TOL

@@ -285,6 +285,25 @@ def test_diagnostic_mode_every_sm_agrees(sizes, B):
         np.testing.assert_array_equal(net.get_weights(), theta.astype(np.float32))
 
 
+@pytest.mark.parametrize("mb", [33, 2])
+def test_deepest_net_the_boundary_allows(mb):
+    """BP_MAX_SIZES layer sizes (8 weight layers) of odd widths, on the
+    persistent kernel (groups of 33) and the one-CTA kernel (groups of 2)."""
+    sizes = (7, 9, 5, 11, 6, 8, 4, 10, 3)
+    assert len(sizes) == bp.BP_MAX_SIZES
+    n = 66
+    X, T, theta = problem(sizes, n, seed=61, lo=-1.0, hi=1.0)
+    st = O.State(sizes, theta, lr=0.3, momentum=0.9)
+    e_ref = O.train_epoch(st, X, T, mb)
+    with bp.Net(sizes, 0.3, 0.9, bp.BP_F32, max_batch=mb) as net:
+        net.set_weights(theta)
+        sse = torch.zeros(len(e_ref), device="cuda")
+        net.train_epoch(dev(X), dev(T), n, mb, sse)
+        net.check()
+        np.testing.assert_allclose(sse.cpu().numpy(), e_ref, rtol=1e-4, atol=1e-6)
+        assert normwise(net.get_weights() - theta, st.theta - theta) <= 1e-4
+
+
 @pytest.mark.parametrize("B", synth.SWEEP_BATCHES)
 def test_batch_sweep_step_matches_oracle(B):
     sizes = (203, 120, 26)
