@@ -39,10 +39,11 @@ constexpr int kWarps = kThreads / 32;
 constexpr int kTU = 8;            // weight-tile rows (output units)
 constexpr int kTJ = 32;           // weight-tile columns (inputs; the bias is the last input)
 constexpr int kPC = 256;          // patterns per staged chunk of the weight phase
-constexpr int kPS = kThreads / (kTJ * kTU / 4);   // pattern splits per tile (8)
 constexpr int kChunkFloats = kPC * (kTU + kTJ);
 constexpr int kNBuf = 3;          // chunk buffers in flight
-constexpr size_t kGradFloats = kNBuf * kChunkFloats + kPS * kTU * kTJ;
+// weight-phase buffers (each chunk: the [kPC][kTJ] activation block, 128-byte
+// swizzled, then the [kPC][kTU] delta block), plus room to align them to 1 KB
+constexpr size_t kGradFloats = kNBuf * kChunkFloats + 256;
 
 constexpr unsigned long long kWaitNs = 2000000000ull;   // 2 s per wait
 constexpr unsigned kWaitIters = 1u << 26;
@@ -528,33 +529,38 @@ struct ChunkPipe {
 // c % kNBuf: the [kPC][kTU] delta block at columns u0 of layer l and the
 // [kPC][kTJ] activation block at columns j0 of layer l - 1.  Thread 0 only.
 // Rows and columns past the ends arrive as zeros.
-__device__ __forceinline__ void issue_chunk(const F32View& v, ChunkPipe& pipe, float* smem, int l,
+__device__ __forceinline__ void issue_chunk(const F32View& v, ChunkPipe& pipe, float* wbuf, int l,
                                             int u0, int j0, int c) {
     const int b = c % kNBuf;
-    float* buf = smem + b * kChunkFloats;
+    float* buf = wbuf + b * kChunkFloats;
     asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_u32(pipe.bar + b)),
                  "r"((unsigned)(kChunkFloats * sizeof(float)))
                  : "memory");
-    tma_load_2d(buf, &v.tm_d[l], u0, c * kPC, pipe.bar + b);
-    tma_load_2d(buf + kPC * kTU, &v.tm_a[l - 1], j0, c * kPC, pipe.bar + b);
+    tma_load_2d(buf, &v.tm_a[l - 1], j0, c * kPC, pipe.bar + b);
+    tma_load_2d(buf + kPC * kTJ, &v.tm_d[l], u0, c * kPC, pipe.bar + b);
 }
 
 // Pooled change of every weight (and bias: the last input column is the true
 // unit's 1) over the B patterns of the group, then either accumulate into G
 // (fused == false) or apply the update directly.  One CTA per 8 x 32 tile;
 // the tile's delta and activation columns stream through shared memory in
-// chunks of kPC patterns by TMA, kNBuf chunks in flight.
+// chunks of kPC patterns by TMA, kNBuf chunks in flight.  Warp w owns a 4 x 4
+// block of the tile (units 4 (w / 8) .., columns 4 (w % 8) ..) and lane l the
+// patterns l, l + 32, ... of every chunk, so each pattern feeds 16 FMAs from
+// two 16-byte loads; the 32 lanes' sums then meet by a butterfly inside the
+// warp.  The activation block arrives 128-byte swizzled by TMA (16-byte chunk
+// k of pattern row p is stored at chunk k ^ (p mod 8)), which keeps the lanes'
+// reads of 32 consecutive rows free of bank conflicts.
 __device__ void weight_phase(const F32View& v, int B, bool fused, bool fold_g, float* smem,
                              ChunkPipe& pipe) {
     const int tid = threadIdx.x;
-    // thread = (pattern split ps, 4 output units uq, input column j)
-    const int ps = tid / (kTJ * kTU / 4), r = tid - ps * (kTJ * kTU / 4);
-    const int uq = r / kTJ, j = r - uq * kTJ;
-    float* red = smem + kNBuf * kChunkFloats;   // [kPS][kTU][kTJ]
+    const int lane = tid & 31, warp = tid >> 5;
+    const int uq = warp >> 3, cq = warp & 7;
+    // 1 KB-aligned base for the swizzled TMA destinations
+    float* wbuf = reinterpret_cast<float*>((reinterpret_cast<uintptr_t>(smem) + 1023) & ~(uintptr_t)1023);
     const int L = v.L;
     const int ntiles = v.tile0[L + 1];
     const int nchunks = (B + kPC - 1) / kPC;
-    constexpr int kPer = kPC / kPS;   // patterns per thread per chunk
     for (int t = blockIdx.x; t < ntiles; t += gridDim.x) {
         int l = 1;
         while (t >= v.tile0[l + 1]) ++l;
@@ -562,21 +568,23 @@ __device__ void weight_phase(const F32View& v, int B, bool fused, bool fold_g, f
         const int tb = lt / v.tcols[l], cb = lt - tb * v.tcols[l];
         const int n_in = v.n[l - 1], n_out = v.n[l];
         const int u0 = tb * kTU, j0 = cb * kTJ;
-        float acc[4] = {0.f, 0.f, 0.f, 0.f};
+        float acc[16];
+#pragma unroll
+        for (int k = 0; k < 16; ++k) acc[k] = 0.f;
         // the buffers' previous contents (weights, pattern rows, the last tile)
         // were read through the generic proxy by every thread before this sync
         __syncthreads();
         if (tid == 0) {
             asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
             asm volatile("fence.proxy.async.global;" ::: "memory");
-            for (int c = 0; c < nchunks && c < kNBuf; ++c) issue_chunk(v, pipe, smem, l, u0, j0, c);
+            for (int c = 0; c < nchunks && c < kNBuf; ++c) issue_chunk(v, pipe, wbuf, l, u0, j0, c);
         }
         for (int c = 0; c < nchunks; ++c) {
             const int b = c % kNBuf;
             mbar_wait(pipe.bar + b, (pipe.parity >> b) & 1u, v.flags);
             pipe.parity ^= 1u << b;
-            float* Ds = smem + b * kChunkFloats;
-            float* As = Ds + kPC * kTU;
+            float* As = wbuf + b * kChunkFloats;
+            float* Ds = As + kPC * kTJ;
             const int pc = B - c * kPC;
             if (pc < kPC) {
                 // rows past the group may hold stale scratch rows: clear them
@@ -584,32 +592,31 @@ __device__ void weight_phase(const F32View& v, int B, bool fused, bool fold_g, f
                 for (int e = tid; e < (kPC - pc) * kTJ; e += kThreads) As[pc * kTJ + e] = 0.f;
                 __syncthreads();
             }
-            const int pp0 = ps * kPer;
 #pragma unroll 4
-            for (int k = 0; k < kPer; ++k) {
-                const int pp = pp0 + k;
-                const float4 d = *reinterpret_cast<const float4*>(Ds + pp * kTU + uq * 4);
-                const float a = As[pp * kTJ + j];
-                acc[0] = fmaf(d.x, a, acc[0]);
-                acc[1] = fmaf(d.y, a, acc[1]);
-                acc[2] = fmaf(d.z, a, acc[2]);
-                acc[3] = fmaf(d.w, a, acc[3]);
+            for (int k = 0; k < kPC / 32; ++k) {
+                const int p = k * 32 + lane;
+                const float4 d = *reinterpret_cast<const float4*>(Ds + p * kTU + uq * 4);
+                const float4 a = *reinterpret_cast<const float4*>(As + p * kTJ + ((cq ^ (p & 7)) << 2));
+                const float dv[4] = {d.x, d.y, d.z, d.w};
+                const float av[4] = {a.x, a.y, a.z, a.w};
+#pragma unroll
+                for (int u = 0; u < 4; ++u)
+#pragma unroll
+                    for (int q = 0; q < 4; ++q) acc[u * 4 + q] = fmaf(dv[u], av[q], acc[u * 4 + q]);
             }
             __syncthreads();
             if (tid == 0 && c + kNBuf < nchunks) {
                 asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-                issue_chunk(v, pipe, smem, l, u0, j0, c + kNBuf);
+                issue_chunk(v, pipe, wbuf, l, u0, j0, c + kNBuf);
             }
         }
-#pragma unroll
-        for (int k = 0; k < 4; ++k) red[(ps * kTU + uq * 4 + k) * kTJ + j] = acc[k];
-        __syncthreads();
-        if (tid < kTU * kTJ) {
-            const int u = tid / kTJ, jj = tid - u * kTJ;
-            float g = 0.f;
-#pragma unroll
-            for (int s = 0; s < kPS; ++s) g += red[(s * kTU + u) * kTJ + jj];
-            const int uu = u0 + u, ii = j0 + jj;
+        // sum over the warp's 32 pattern lanes (fixed order): afterwards lane s
+        // (s < 16) holds value s = (unit u, column q) = (s / 4, s % 4)
+        reduce_scatter<16>(acc, lane);
+        const float g0 = acc[0] + __shfl_xor_sync(0xffffffffu, acc[0], 16);
+        if (lane < 16) {
+            float g = g0;
+            const int uu = u0 + uq * 4 + (lane >> 2), ii = j0 + cq * 4 + (lane & 3);
             if (uu < n_out && ii <= n_in) {
                 const long long idx = v.woff[l] + (long long)uu * v.kp[l] + ii;   // ii == n_in: bias
                 if (!fused) {
@@ -1065,7 +1072,8 @@ int f32_max_pg(const int* n, int L) {
 
 // One float32 2-D map over rows [rows][pitch] (pitch floats apart), boxes of
 // box_cols x kPC, zero fill outside.
-static bool encode_rows(CUtensorMap* map, const float* base, int rows, int pitch, int box_cols) {
+static bool encode_rows(CUtensorMap* map, const float* base, int rows, int pitch, int box_cols,
+                        CUtensorMapSwizzle swizzle = CU_TENSOR_MAP_SWIZZLE_NONE) {
     PFN_cuTensorMapEncodeTiled_v12000 enc = tensor_map_encoder();
     if (enc == nullptr) return false;
     cuuint64_t dims[2] = {(cuuint64_t)pitch, (cuuint64_t)rows};
@@ -1073,14 +1081,15 @@ static bool encode_rows(CUtensorMap* map, const float* base, int rows, int pitch
     cuuint32_t box[2] = {(cuuint32_t)box_cols, (cuuint32_t)kPC};
     cuuint32_t estr[2] = {1, 1};
     return enc(map, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 2, const_cast<float*>(base), dims, strides, box,
-               estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE,
+               estr, CU_TENSOR_MAP_INTERLEAVE_NONE, swizzle,
                CU_TENSOR_MAP_L2_PROMOTION_L2_128B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
 cudaError_t f32_maps(F32View& v) {
     for (int l = 1; l <= v.L; ++l) {
         if (!encode_rows(&v.tm_d[l], v.D + v.doff[l], v.cap, v.dpitch[l], kTU) ||
-            !encode_rows(&v.tm_a[l - 1], v.A + v.aoff[l - 1], v.cap, v.apitch[l - 1], kTJ))
+            !encode_rows(&v.tm_a[l - 1], v.A + v.aoff[l - 1], v.cap, v.apitch[l - 1], kTJ,
+                         CU_TENSOR_MAP_SWIZZLE_128B))
             return cudaErrorInvalidValue;
     }
     return cudaSuccess;
