@@ -480,6 +480,8 @@ bp_status bp_check(bp_net* net, void* stream) {
         BP_CUDA(cudaMemset(net->bar, 0, (size_t)bp::kBarWords * sizeof(unsigned)), "bp_check");
     if (flags & kFlagTimeout)
         return fail(BP_ETIMEOUT, "a bounded device-side wait ran out; the launch stopped early");
+    if (flags & kFlagBounds)
+        return fail(BP_ESTATE, "a bounds check of the checked build failed; the phase was skipped");
     return fail(BP_ENONFINITE, "the summed squared error of a group was not finite");
 }
 

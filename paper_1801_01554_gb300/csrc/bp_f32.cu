@@ -51,6 +51,30 @@ constexpr unsigned kWaitIters = 1u << 26;
 // ------------------------------------------------------------ small helpers
 __device__ __forceinline__ float sigmoid_f(float x) { return 1.0f / (1.0f + expf(-x)); }
 
+// Checked build (-DBP_CHECK): phases test that their shared-memory regions fit
+// the launch's dynamic shared memory and that their rows and tile origins lie
+// inside their buffers; a failed test latches kFlagBounds (bp_check reports it)
+// and the phase skips its accesses.  Without BP_CHECK the tests compile away.
+extern __shared__ __align__(128) float g_dyn_smem[];   // every kernel's dynamic shared memory
+__device__ __forceinline__ const float* pattern_smem_base() { return g_dyn_smem; }
+__device__ __forceinline__ unsigned dyn_smem_floats() {
+    unsigned b;
+    asm("mov.u32 %0, %%dynamic_smem_size;" : "=r"(b));
+    return b / 4;
+}
+__device__ __forceinline__ bool bounds_ok(bool ok, int* flags) {
+#ifdef BP_CHECK
+    if (!ok) {
+        atomicOr(flags, kFlagBounds);
+        return false;
+    }
+#else
+    (void)ok;
+    (void)flags;
+#endif
+    return true;
+}
+
 // Table-lookup logistic (Section 4.3, Figure 3): the logistic at 256 equally
 // spaced points over [-15, 15], built in shared memory by each CTA that runs a
 // forward pass with the table mode on.  Inputs outside the range take the end
@@ -418,6 +442,12 @@ __device__ float pattern_phase(const F32View& v, const PatLayout& q, const float
     float sse = 0.f;
     const int q_lo = whole ? 0 : (int)((long long)B * blockIdx.x / gridDim.x);
     const int q_hi = whole ? B : (int)((long long)B * (blockIdx.x + 1) / gridDim.x);
+    if (!bounds_ok((size_t)(smem - pattern_smem_base()) + q.total <= dyn_smem_floats() &&
+                       ((!to_scratch && do_fwd) || B <= v.cap),
+                   v.flags)) {
+        if (wc != nullptr) stage_weights_wait(*wc, v.flags);
+        return block_sum(0.f);
+    }
     for (int p0 = q_lo; p0 < q_hi; p0 += PG) {
         const int np = min(PG, q_hi - p0);
         if (!(rows_issued && p0 == q_lo))
@@ -561,6 +591,10 @@ __device__ void weight_phase(const F32View& v, int B, bool fused, bool fold_g, f
     const int L = v.L;
     const int ntiles = v.tile0[L + 1];
     const int nchunks = (B + kPC - 1) / kPC;
+    if (!bounds_ok((size_t)(wbuf - pattern_smem_base()) + kNBuf * kChunkFloats <= dyn_smem_floats() &&
+                       B <= v.cap,
+                   v.flags))
+        return;
     for (int t = blockIdx.x; t < ntiles; t += gridDim.x) {
         int l = 1;
         while (t >= v.tile0[l + 1]) ++l;
@@ -568,6 +602,9 @@ __device__ void weight_phase(const F32View& v, int B, bool fused, bool fold_g, f
         const int tb = lt / v.tcols[l], cb = lt - tb * v.tcols[l];
         const int n_in = v.n[l - 1], n_out = v.n[l];
         const int u0 = tb * kTU, j0 = cb * kTJ;
+        // TMA origins: columns 16-byte aligned and inside the row pitches
+        if (!bounds_ok(u0 % 4 == 0 && j0 % 4 == 0 && u0 < v.dpitch[l] && j0 < v.apitch[l - 1], v.flags))
+            return;
         float acc[16];
 #pragma unroll
         for (int k = 0; k < 16; ++k) acc[k] = 0.f;
@@ -676,6 +713,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     __syncthreads();
     if (WS) {
         mbar_init1(&s_bar);
+        if (!bounds_ok((unsigned)v.wsm <= dyn_smem_floats(), v.flags)) return;
         stage_weights(v.theta, v.P, smem, &s_bar, phase, v.flags);
         pattern_phase<PG>(v, q, smem, X, nullptr, B, true, false, Y, pattern_base<true>(v, smem));
     } else {
@@ -692,6 +730,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     float e;
     if (WS) {
         mbar_init1(&s_bar);
+        if (!bounds_ok((unsigned)v.wsm <= dyn_smem_floats(), v.flags)) return;
         stage_weights(v.theta, v.P, smem, &s_bar, phase, v.flags);
         e = pattern_phase<PG>(v, q, smem, nullptr, T, B, false, true, nullptr, pattern_base<true>(v, smem));
     } else {
@@ -712,6 +751,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     unsigned phase = 0;
     sigmoid_table_init(v);
     mbar_init1(&s_bar);
+    if (WS && !bounds_ok((unsigned)v.wsm <= dyn_smem_floats(), v.flags)) return;
     float e;
     if (WS) {
         stage_weights(v.theta, v.P, smem, &s_bar, phase, v.flags);
@@ -769,6 +809,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     unsigned target = __ldcg(v.bar);
     const int n0 = v.n[0], nL = v.n[v.L];
     float* pat = pattern_base<WS>(v, smem);
+    if (WS && !bounds_ok((unsigned)v.wsm <= dyn_smem_floats(), v.flags)) return;
     for (int s = 0; s < n_steps; ++s) {
         const long long p0 = (long long)s * minibatch;
         const int B = (int)min((long long)minibatch, (long long)n_patterns - p0);
@@ -825,6 +866,9 @@ __global__ void __launch_bounds__(kThreads, 1)
     mbar_init1(&s_bar);
     float* pat[2] = {smem + v.wsm, smem + v.wsm + q.total};
     const int n0 = v.n[0], nL = v.n[v.L];
+    if (!bounds_ok((unsigned)v.wsm + 2u * (unsigned)q.total <= dyn_smem_floats() && minibatch <= PG,
+                   v.flags))
+        return;
     // slot m of this thread: layer lm, row jm (or -1), float4 column cm
     float4 vel[NV4];
 #pragma unroll

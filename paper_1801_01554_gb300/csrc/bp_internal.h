@@ -15,6 +15,7 @@ constexpr int kMaxL = BP_MAX_SIZES - 1;   // weight layers
 // Bits of the device-side error word latched by kernels.
 constexpr int kFlagTimeout = 1;     // a bounded wait ran out
 constexpr int kFlagNonfinite = 2;   // an error sum was NaN/Inf
+constexpr int kFlagBounds = 4;      // a check of the checked build (-DBP_CHECK) failed
 
 // Words of the grid-barrier state (two used, padded to 16 bytes).
 constexpr int kBarWords = 4;
