@@ -2,27 +2,31 @@
 //
 // One training step over a group of B patterns runs in two phases:
 //
-//   pattern phase (case-parallel, Section 4.1): every CTA first copies all the
+//   pattern phase (case-parallel, Section 4.1): every CTA copies all the
 //     weights into its shared memory with one bulk copy (they fit for the
-//     NETtalk-sized nets of Section 6.3; larger nets read them from L2), then
-//     runs the whole net on its share of the patterns: forward pass (Section 3),
-//     output delta (t-o)o(1-o) with the summed squared error, hidden deltas
-//     (W^T delta) h(1-h) for every hidden layer and none for the inputs
-//     (Section 6.1).  Dot products are summed as a binary tree across the
-//     warp (Section 10.3).  Activations (with a trailing 1 for the bias input)
-//     and deltas go to scratch rows aligned to 16 bytes.
+//     NETtalk-sized nets of Section 6.3; larger nets read them from L2), while
+//     its first input and target rows arrive, then runs the whole net on its
+//     share of the patterns: forward pass (Section 3), output delta (t-o)o(1-o)
+//     with the summed squared error, hidden deltas (W^T delta) h(1-h) for every
+//     hidden layer and none for the inputs (Section 6.1).  Weights are kept as
+//     padded rows [W | b | 0..] and activations with a trailing 1, so a row
+//     product is a unit's net input with its bias; the forward pass sums each
+//     dot product as a binary tree across a lane group (Section 10.3).
+//     Activation and delta rows go to scratch rows aligned to 16 bytes.
 //
 //   weight phase (Section 5's "bundle" of weights processed over the whole
-//     group of cases): one CTA per 8 x 32 tile of [W_l | b_l] stages the
-//     group's deltas and activations through shared memory with 16-byte
-//     cp.async, sums delta[p,j] a[p,i] over all patterns with 4-wide register
-//     blocking (Sections 3, 4.1), then either accumulates into G (bp_backward)
-//     or applies the momentum update of Section 6.2.1 at once (training), so the
-//     pooled change never goes to memory.
+//     group of cases): one CTA per 8 x 32 tile of [W_l | b_l] streams the
+//     group's deltas and activations through shared memory with 2-D TMA loads,
+//     sums delta[p,j] a[p,i] over all patterns with 4 x 4 register blocks per
+//     lane and a warp butterfly (Sections 3, 4.1), then either accumulates into
+//     G (bp_backward) or applies the momentum update of Section 6.2.1 at once
+//     (training), so the pooled change never goes to memory.
 //
 // A training launch is a persistent cooperative kernel that loops over any
 // number of groups with a grid barrier between the phases; every wait in the
-// barrier is bounded and latches kFlagTimeout instead of hanging.
+// barrier is bounded and latches kFlagTimeout instead of hanging.  Groups of at
+// most 4 patterns run on one CTA instead (k_train_small), with the weights
+// resident in its shared memory for the whole launch.
 #include <cuda_runtime.h>
 
 #include <algorithm>
