@@ -214,10 +214,10 @@ bp_status bp_check(bp_net* net, void* stream);
  *   device array of 8 MiB, which every GPU that loads the library holds until the
  *   process exits.  Sizes whose scratch exceeds it are rejected with
  *   BP_EINVAL; the scratch takes 4 * (8 + roundup4(SMs) + 2 * Q + minibatch *
- *   (sum over l = 0..L of roundup4(n_l + 1) + sum over l = 1..L of roundup4(n_l)))
+ *   (sum over l = 0..L of roundup32(n_l + 1) + sum over l = 1..L of roundup8(n_l)))
  *   bytes, where Q = sum over l = 1..L of n_l * roundup4(n_{l-1} + 1) holds a
  *   copy of the weights and of the weight changes in the kernel's row layout
- *   (for 203-120-26 on 152 SMs a minibatch of up to 4,050 patterns fits).
+ *   (for 203-120-26 on 152 SMs a minibatch of up to 3,808 patterns fits).
  *   The first call on a device looks up the array's device address and sets
  *   kernel attributes; make that first call before any stream capture.  All
  *   calls on a device share the array and find the previous call's contents:

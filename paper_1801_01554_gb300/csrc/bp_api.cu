@@ -216,8 +216,6 @@ bp_status bp_create(const int* sizes, int n_layers, float lr, float momentum, in
         v.G = net->G;
         v.A = net->A;
         v.D = net->D;
-        e = f32_maps(v);
-        if (e != cudaSuccess) return bail(cuda_fail(e, "cuTensorMapEncodeTiled(scratch)"));
         v.sse_part = net->sse_part;
         v.bar = net->bar;
         v.flags = net->flags;

@@ -404,17 +404,32 @@ __device__ void hidden_delta(const float* Wn, int kpn, int n, int nn, const floa
     }
 }
 
-// Copies np rows of `pitch` floats (a multiple of 4) from shared to global
-// memory as float4.
-template <int PG>
-__device__ __forceinline__ void rows_to_global(float* dst, const float* src, int pitch, int np) {
+// Scratch addresses (see F32View): float4 chunk k (columns 4k .. 4k + 3) of
+// pattern p's activations of layer l, and of its deltas.
+__device__ __forceinline__ float4* act_chunk(const F32View& v, int l, long long p, int k) {
+    return reinterpret_cast<float4*>(v.A + v.aoff[l] + (long long)(k >> 3) * v.cap * 32 + p * 32) +
+           ((k & 7) ^ (int)(p & 7));
+}
+__device__ __forceinline__ float4* delta_chunk(const F32View& v, int l, long long p, int k) {
+    return reinterpret_cast<float4*>(v.D + v.doff[l] + (long long)(k >> 1) * v.cap * 8 + p * 8) +
+           ((k & 1) ^ (int)((p >> 2) & 1));
+}
+
+// Writes np rows (pitch floats apart in shared memory) of layer l's
+// activations (or deltas) to the blocked scratch layout; chunks past the row
+// pitch are written as zeros so that every block column is defined.
+template <int PG, bool DELTA>
+__device__ __forceinline__ void rows_to_scratch(const F32View& v, int l, const float* src, int pitch,
+                                                int p0, int np) {
     constexpr int TP = kThreads / PG;
     const int p = threadIdx.x / TP, c0 = threadIdx.x % TP;
     if (p < np) {
-        const int q4 = pitch >> 2;
-        float4* d = reinterpret_cast<float4*>(dst + (size_t)p * pitch);
-        const float4* s = reinterpret_cast<const float4*>(src + p * pitch);
-        for (int c = c0; c < q4; c += TP) d[c] = s[c];
+        const int q4 = pitch >> 2, nk = DELTA ? 2 * v.dtb[l] : 8 * v.acb[l];
+        for (int k = c0; k < nk; k += TP) {
+            const float4 x = k < q4 ? reinterpret_cast<const float4*>(src + p * pitch)[k]
+                                    : make_float4(0.f, 0.f, 0.f, 0.f);
+            *(DELTA ? delta_chunk(v, l, p0 + p, k) : act_chunk(v, l, p0 + p, k)) = x;
+        }
     }
 }
 
@@ -460,11 +475,9 @@ __device__ float pattern_phase(const F32View& v, const PatLayout& q, const float
             // activations of the last forward, reloaded from scratch
             for (int l = 1; l <= L; ++l) {
                 const int ap = v.apitch[l], q4 = ap >> 2;
-                const float4* src =
-                    reinterpret_cast<const float4*>(v.A + v.aoff[l] + (size_t)(p0 + pr) * ap);
                 float4* dst = reinterpret_cast<float4*>(smem + q.sa[l] + pr * ap);
                 for (int c = c0; c < q4; c += TP)
-                    dst[c] = (pr < np) ? __ldcg(src + c) : make_float4(0.f, 0.f, 0.f, 0.f);
+                    dst[c] = (pr < np) ? __ldcg(act_chunk(v, l, p0 + pr, c)) : make_float4(0.f, 0.f, 0.f, 0.f);
             }
         }
         if (wc != nullptr) {
@@ -481,8 +494,7 @@ __device__ float pattern_phase(const F32View& v, const PatLayout& q, const float
             }
             // activation rows, bias column and pads included
             for (int l = 0; l <= L && to_scratch; ++l)
-                rows_to_global<PG>(v.A + v.aoff[l] + (size_t)p0 * v.apitch[l], smem + q.sa[l],
-                                   v.apitch[l], np);
+                rows_to_scratch<PG, false>(v, l, smem + q.sa[l], v.apitch[l], p0, np);
             if (Y != nullptr && pr < np) {
                 for (int k = c0; k < nL; k += TP)
                     Y[(size_t)(p0 + pr) * nL + k] = smem[q.sa[L] + pr * v.apitch[L] + k];
@@ -512,8 +524,7 @@ __device__ float pattern_phase(const F32View& v, const PatLayout& q, const float
                 __syncthreads();
             }
             for (int l = 1; l <= L && to_scratch; ++l)
-                rows_to_global<PG>(v.D + v.doff[l] + (size_t)p0 * v.dpitch[l], smem + q.sd[l],
-                                   v.dpitch[l], np);
+                rows_to_scratch<PG, true>(v, l, smem + q.sd[l], v.dpitch[l], p0, np);
         }
         __syncthreads();
     }
@@ -542,13 +553,11 @@ __device__ __forceinline__ float guard_count(float guard, float g, unsigned& n_b
 }
 
 
-__device__ __forceinline__ void tma_load_2d(float* smem_dst, const CUtensorMap* map, int c0, int c1,
-                                            uint64_t* bar) {
-    asm volatile(
-        "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes "
-        "[%0], [%1, {%2, %3}], [%4];" ::"r"(smem_u32(smem_dst)),
-        "l"((unsigned long long)map), "r"(c0), "r"(c1), "r"(smem_u32(bar))
-        : "memory");
+__device__ __forceinline__ void bulk_load(float* smem_dst, const float* src, unsigned bytes, uint64_t* bar) {
+    asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::
+                     "r"(smem_u32(smem_dst)),
+                 "l"(src), "r"(bytes), "r"(smem_u32(bar))
+                 : "memory");
 }
 
 // Weight-phase pipeline state of a CTA: kNBuf chunk buffers, each filled by two
@@ -559,38 +568,39 @@ struct ChunkPipe {
     unsigned parity;
 };
 
-// Issues chunk c of a tile (patterns [c * kPC, c * kPC + kPC)) into buffer
-// c % kNBuf: the [kPC][kTU] delta block at columns u0 of layer l and the
-// [kPC][kTJ] activation block at columns j0 of layer l - 1.  Thread 0 only.
-// Rows and columns past the ends arrive as zeros.
+// Issues chunk c of a tile (patterns [c * kPC, c * kPC + rows)) into buffer
+// c % kNBuf: the [rows][kTJ] activation block cb of layer l - 1, then the
+// [rows][kTU] delta block tb of layer l, each one contiguous bulk copy from the
+// blocked scratch.  Thread 0 only.
 __device__ __forceinline__ void issue_chunk(const F32View& v, ChunkPipe& pipe, float* wbuf, int l,
-                                            int u0, int j0, int c) {
+                                            int tb, int cb, int c, int rows) {
     const int b = c % kNBuf;
     float* buf = wbuf + b * kChunkFloats;
+    const unsigned abytes = (unsigned)rows * kTJ * 4, dbytes = (unsigned)rows * kTU * 4;
     asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_u32(pipe.bar + b)),
-                 "r"((unsigned)(kChunkFloats * sizeof(float)))
+                 "r"(abytes + dbytes)
                  : "memory");
-    tma_load_2d(buf, &v.tm_a[l - 1], j0, c * kPC, pipe.bar + b);
-    tma_load_2d(buf + kPC * kTJ, &v.tm_d[l], u0, c * kPC, pipe.bar + b);
+    const long long p0 = (long long)c * kPC;
+    bulk_load(buf, v.A + v.aoff[l - 1] + (long long)cb * v.cap * kTJ + p0 * kTJ, abytes, pipe.bar + b);
+    bulk_load(buf + kPC * kTJ, v.D + v.doff[l] + (long long)tb * v.cap * kTU + p0 * kTU, dbytes, pipe.bar + b);
 }
 
 // Pooled change of every weight (and bias: the last input column is the true
 // unit's 1) over the B patterns of the group, then either accumulate into G
 // (fused == false) or apply the update directly.  One CTA per 8 x 32 tile;
-// the tile's delta and activation columns stream through shared memory in
-// chunks of kPC patterns by TMA, kNBuf chunks in flight.  Warp w owns a 4 x 4
-// block of the tile (units 4 (w / 8) .., columns 4 (w % 8) ..) and lane l the
-// patterns l, l + 32, ... of every chunk, so each pattern feeds 16 FMAs from
-// two 16-byte loads; the 32 lanes' sums then meet by a butterfly inside the
-// warp.  The activation block arrives 128-byte swizzled by TMA (16-byte chunk
-// k of pattern row p is stored at chunk k ^ (p mod 8)), which keeps the lanes'
-// reads of 32 consecutive rows free of bank conflicts.
+// the tile's delta and activation blocks stream through shared memory in
+// chunks of kPC patterns, one bulk copy each from the blocked scratch, kNBuf
+// chunks in flight.  Warp w owns a 4 x 4 block of the tile (units 4 (w / 8) ..,
+// columns 4 (w % 8) ..) and lane l the patterns l, l + 32, ... of every chunk,
+// so each pattern feeds 16 FMAs from two 16-byte loads; the 32 lanes' sums then
+// meet by a butterfly inside the warp.  The blocks' row chunks are stored
+// permuted by pattern (see F32View), which keeps the lanes' reads of 32
+// consecutive rows free of bank conflicts.
 __device__ void weight_phase(const F32View& v, int B, bool fused, bool fold_g, float* smem,
                              ChunkPipe& pipe) {
     const int tid = threadIdx.x;
     const int lane = tid & 31, warp = tid >> 5;
     const int uq = warp >> 3, cq = warp & 7;
-    // 1 KB-aligned base for the swizzled TMA destinations
     float* wbuf = reinterpret_cast<float*>((reinterpret_cast<uintptr_t>(smem) + 1023) & ~(uintptr_t)1023);
     const int L = v.L;
     const int ntiles = v.tile0[L + 1];
@@ -606,9 +616,8 @@ __device__ void weight_phase(const F32View& v, int B, bool fused, bool fold_g, f
         const int tb = lt / v.tcols[l], cb = lt - tb * v.tcols[l];
         const int n_in = v.n[l - 1], n_out = v.n[l];
         const int u0 = tb * kTU, j0 = cb * kTJ;
-        // TMA origins: columns 16-byte aligned and inside the row pitches
-        if (!bounds_ok(u0 % 4 == 0 && j0 % 4 == 0 && u0 < v.dpitch[l] && j0 < v.apitch[l - 1], v.flags))
-            return;
+        // the tile's blocks exist in the scratch layout
+        if (!bounds_ok(tb < v.dtb[l] && cb < v.acb[l - 1], v.flags)) return;
         float acc[16];
 #pragma unroll
         for (int k = 0; k < 16; ++k) acc[k] = 0.f;
@@ -618,7 +627,8 @@ __device__ void weight_phase(const F32View& v, int B, bool fused, bool fold_g, f
         if (tid == 0) {
             asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
             asm volatile("fence.proxy.async.global;" ::: "memory");
-            for (int c = 0; c < nchunks && c < kNBuf; ++c) issue_chunk(v, pipe, wbuf, l, u0, j0, c);
+            for (int c = 0; c < nchunks && c < kNBuf; ++c)
+                issue_chunk(v, pipe, wbuf, l, tb, cb, c, min(kPC, B - c * kPC));
         }
         for (int c = 0; c < nchunks; ++c) {
             const int b = c % kNBuf;
@@ -636,7 +646,7 @@ __device__ void weight_phase(const F32View& v, int B, bool fused, bool fold_g, f
 #pragma unroll 4
             for (int k = 0; k < kPC / 32; ++k) {
                 const int p = k * 32 + lane;
-                const float4 d = *reinterpret_cast<const float4*>(Ds + p * kTU + uq * 4);
+                const float4 d = *reinterpret_cast<const float4*>(Ds + p * kTU + ((uq ^ ((p >> 2) & 1)) << 2));
                 const float4 a = *reinterpret_cast<const float4*>(As + p * kTJ + ((cq ^ (p & 7)) << 2));
                 const float dv[4] = {d.x, d.y, d.z, d.w};
                 const float av[4] = {a.x, a.y, a.z, a.w};
@@ -648,7 +658,7 @@ __device__ void weight_phase(const F32View& v, int B, bool fused, bool fold_g, f
             __syncthreads();
             if (tid == 0 && c + kNBuf < nchunks) {
                 asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-                issue_chunk(v, pipe, wbuf, l, u0, j0, c + kNBuf);
+                issue_chunk(v, pipe, wbuf, l, tb, cb, c + kNBuf, min(kPC, B - (c + kNBuf) * kPC));
             }
         }
         // sum over the warp's 32 pattern lanes (fixed order): afterwards lane s
@@ -1037,8 +1047,9 @@ long long f32_layout(F32View& v, const int* n, int L, int cap) {
     v.tile0[0] = v.tile0[1] = 0;
     for (int l = 0; l <= L; ++l) {
         v.apitch[l] = (n[l] + 1 + 3) & ~3;
+        v.acb[l] = (n[l] + 1 + kTJ - 1) / kTJ;
         v.aoff[l] = a;
-        a += (long long)cap * v.apitch[l];
+        a += (long long)cap * v.acb[l] * kTJ;
     }
     long long pp = 0;
     for (int l = 1; l <= L; ++l) {
@@ -1050,8 +1061,9 @@ long long f32_layout(F32View& v, const int* n, int L, int cap) {
         v.pb[l] = pp;
         pp += n[l];
         v.dpitch[l] = (n[l] + 3) & ~3;
+        v.dtb[l] = (n[l] + kTU - 1) / kTU;
         v.doff[l] = d;
-        d += (long long)cap * v.dpitch[l];
+        d += (long long)cap * v.dtb[l] * kTU;
         const int rows = (n[l] + kTU - 1) / kTU, cols = (n[l - 1] + 1 + kTJ - 1) / kTJ;
         v.tcols[l] = cols;
         v.tile0[l] = tiles;
@@ -1116,31 +1128,6 @@ int f32_max_pg(const int* n, int L) {
     for (int pg = 1; pg <= 8; pg *= 2)
         if (f32_smem_bytes(n, L, pg) <= kSmemLimit) best = pg;
     return best;
-}
-
-// One float32 2-D map over rows [rows][pitch] (pitch floats apart), boxes of
-// box_cols x kPC, zero fill outside.
-static bool encode_rows(CUtensorMap* map, const float* base, int rows, int pitch, int box_cols,
-                        CUtensorMapSwizzle swizzle = CU_TENSOR_MAP_SWIZZLE_NONE) {
-    PFN_cuTensorMapEncodeTiled_v12000 enc = tensor_map_encoder();
-    if (enc == nullptr) return false;
-    cuuint64_t dims[2] = {(cuuint64_t)pitch, (cuuint64_t)rows};
-    cuuint64_t strides[1] = {(cuuint64_t)pitch * sizeof(float)};
-    cuuint32_t box[2] = {(cuuint32_t)box_cols, (cuuint32_t)kPC};
-    cuuint32_t estr[2] = {1, 1};
-    return enc(map, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 2, const_cast<float*>(base), dims, strides, box,
-               estr, CU_TENSOR_MAP_INTERLEAVE_NONE, swizzle,
-               CU_TENSOR_MAP_L2_PROMOTION_L2_128B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
-}
-
-cudaError_t f32_maps(F32View& v) {
-    for (int l = 1; l <= v.L; ++l) {
-        if (!encode_rows(&v.tm_d[l], v.D + v.doff[l], v.cap, v.dpitch[l], kTU) ||
-            !encode_rows(&v.tm_a[l - 1], v.A + v.aoff[l - 1], v.cap, v.apitch[l - 1], kTJ,
-                         CU_TENSOR_MAP_SWIZZLE_128B))
-            return cudaErrorInvalidValue;
-    }
-    return cudaSuccess;
 }
 
 template <int PG, bool GUARD>

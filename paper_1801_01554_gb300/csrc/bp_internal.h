@@ -28,10 +28,16 @@ constexpr int kBarWords = 4;
 //              (also the size of its shared-memory copy, wsm).  The API's
 //              packed layout (W_l row-major, then b_l; Pp floats) is converted
 //              on the way in and out.
-//   A: activation rows of layers 0..L, layer l at aoff[l] with pitch apitch[l]
-//      = n_l + 1 rounded up to 4 (column n_l holds the true unit's 1).
-//   D: delta rows of layers 1..L at doff[l], pitch dpitch[l] = n_l rounded up to 4.
-//   Both hold `cap` patterns.
+//   A: activations of layers 0..L for `cap` patterns, layer l at aoff[l] in
+//      acb[l] column blocks of [cap][32] floats (columns 32b .. 32b + 31;
+//      column n_l holds the true unit's 1, columns past it are 0).  Inside a
+//      pattern's 128-byte block row the 16-byte chunk k sits at k ^ (p mod 8),
+//      so that the weight phase's lanes read 32 consecutive rows without bank
+//      conflicts; a chunk of a tile is one contiguous bulk copy.
+//   D: deltas of layers 1..L at doff[l] in dtb[l] blocks of [cap][8] floats,
+//      chunk k of a 32-byte block row at k ^ ((p / 4) mod 2).
+//   apitch[l] = n_l + 1 and dpitch[l] = n_l rounded up to 4 are the row
+//   pitches of the same rows in shared memory.
 //   Gradient tiles: layer l owns tiles [tile0[l], tile0[l+1]) of 8 rows x 32
 //   columns of the [n_l, n_{l-1} + 1] matrix (last column = bias).
 struct F32View {
@@ -47,6 +53,8 @@ struct F32View {
     int wsm;
     int apitch[BP_MAX_SIZES];
     int dpitch[BP_MAX_SIZES];
+    int acb[BP_MAX_SIZES];         // 32-column blocks of layer l's activations
+    int dtb[BP_MAX_SIZES];         // 8-column blocks of layer l's deltas
     long long aoff[BP_MAX_SIZES];
     long long doff[BP_MAX_SIZES];
     long long a_floats, d_floats;
@@ -64,13 +72,6 @@ struct F32View {
     int sig_table;        // 1: table-lookup logistic (Section 4.3) in the forward pass
     float guard;          // > 0: fault guard of Section 8 (|change| > guard is zeroed)
     unsigned* faults;     // changes the guard zeroed (flags[1])
-    // TMA maps of the weight phase (f32_maps): tm_d[l] over the delta rows of
-    // layer l (boxes of 8 columns x 256 patterns), tm_a[l] over the activation
-    // rows of layer l (boxes of 32 columns x 256 patterns); zero fill past the
-    // row pitch and past `cap`.  Kernels take the view as a __grid_constant__
-    // parameter so that the maps can be addressed in place.
-    CUtensorMap tm_d[BP_MAX_SIZES];
-    CUtensorMap tm_a[BP_MAX_SIZES];
 };
 
 // Offsets (floats, each a multiple of 4) of a CTA's pattern buffers for PG
@@ -103,8 +104,6 @@ long long f32_layout(F32View& v, const int* n, int L, int cap);
 int f32_max_pg(const int* n, int L);
 size_t f32_smem_bytes(const int* n, int L, int pg);
 cudaError_t f32_setup(int device);   // opt-in shared memory limits, once per process
-// Encodes the TMA maps of v over its A and D buffers (set A, D and the layout first).
-cudaError_t f32_maps(F32View& v);
 F32Plan f32_plan(const F32View& v, int batch, int num_sms);
 
 cudaError_t f32_forward(const F32View& v, const float* X, int batch, float* Y,

@@ -125,10 +125,6 @@ extern "C" bp_status bp_train_epoch_noalloc(const int* layer_sizes, int n_layers
     float* V_pad = theta_pad + v.P;
     v.A = base + head;
     v.D = base + head + v.a_floats;
-    if (f32_maps(v) != cudaSuccess) {
-        set_error_message("bp_train_epoch_noalloc: cuTensorMapEncodeTiled failed for the scratch");
-        return BP_ECUDA;
-    }
     // the kernel works on padded copies of the caller's (packed) weights and
     // weight changes, copied back when it is done
     v.theta = theta_pad;
