@@ -618,6 +618,16 @@ __device__ void weight_phase(const F32View& v, int B, bool fused, bool fold_g, f
         const int u0 = tb * kTU, j0 = cb * kTJ;
         // the tile's blocks exist in the scratch layout
         if (!bounds_ok(tb < v.dtb[l] && cb < v.acb[l - 1], v.flags)) return;
+        // this lane's output (lanes 0..15 of each warp) and its current weight
+        // state, loaded now so that their latency hides behind the chunks
+        const int uu = u0 + uq * 4 + ((lane & 15) >> 2), ii = j0 + cq * 4 + (lane & 3);
+        const bool mine = lane < 16 && uu < n_out && ii <= n_in;
+        const long long idx = v.woff[l] + (long long)uu * v.kp[l] + ii;   // ii == n_in: bias
+        float v_old = 0.f, g_old = 0.f;
+        if (mine) {
+            if (fused) v_old = __ldcg(v.V + idx);
+            if (!fused || fold_g) g_old = __ldcg(v.G + idx);
+        }
         float acc[16];
 #pragma unroll
         for (int k = 0; k < 16; ++k) acc[k] = 0.f;
@@ -667,18 +677,16 @@ __device__ void weight_phase(const F32View& v, int B, bool fused, bool fold_g, f
         const float g0 = acc[0] + __shfl_xor_sync(0xffffffffu, acc[0], 16);
         if (lane < 16) {
             float g = g0;
-            const int uu = u0 + uq * 4 + (lane >> 2), ii = j0 + cq * 4 + (lane & 3);
-            if (uu < n_out && ii <= n_in) {
-                const long long idx = v.woff[l] + (long long)uu * v.kp[l] + ii;   // ii == n_in: bias
+            if (mine) {
                 if (!fused) {
-                    v.G[idx] += g;
+                    v.G[idx] = g_old + g;
                 } else {
                     if (fold_g) {
-                        g += v.G[idx];
+                        g += g_old;
                         v.G[idx] = 0.f;
                     }
                     g = guard_change(v, g);
-                    const float vel = v.lr * v.grad_scale * g + v.momentum * v.V[idx];
+                    const float vel = v.lr * v.grad_scale * g + v.momentum * v_old;
                     v.V[idx] = vel;
                     v.theta[idx] += vel;
                 }
