@@ -194,12 +194,12 @@ def time_oracle(patterns_cap, budget_s, steps=1, warmup=0, min_s=0.0, max_epochs
 
 
 # DRAM bytes per pattern of the float32 training kernel on the 203-120-26
-# workload: 15,545,856 bytes (15,290,624 read + 255,232 written) in one ncu
+# workload: 15,513,856 bytes (15,293,952 read + 219,904 written) in one ncu
 # capture of the timed k_train launch of `bench.py --patterns 16384` (16,384
 # patterns after an L2 flush; profiles/k_train_nettalk120_launches.md).  The
 # inputs and targets are read once (916 bytes per pattern); everything else
 # stays in L2.  Re-measure after any change to the kernel.
-K_TRAIN_DRAM_BYTES_PER_PATTERN = 15_545_856 / 16_384
+K_TRAIN_DRAM_BYTES_PER_PATTERN = 15_513_856 / 16_384
 
 
 def connections(sizes):

@@ -83,14 +83,14 @@ class GB300Phases:
     for the 203-120-26 net with each phase looped inside one launch."""
     n_sm: int = 152
     barrier_us: float = 1.29          # one grid barrier (two per update)
-    weight_copy_us: float = 0.71      # 110.8 KB bulk copy into each CTA's shared memory
+    weight_copy_us: float = 0.70      # 110.8 KB bulk copy into each CTA's shared memory
     # one pattern pass of PG patterns on a CTA (rows, forward, deltas, rows out)
-    pass_us: tuple = ((1, 4.05), (2, 4.34), (4, 5.21), (8, 7.70))
-    chunk_us: float = 0.96            # one 256-pattern chunk of a weight tile
-    weight_fixed_us: float = 1.17     # chunk issue, tile reduction and update
-    skew_us: float = 1.68             # arrival skew between CTAs, the remainder at B = 512
+    pass_us: tuple = ((1, 4.11), (2, 4.44), (4, 5.30), (8, 7.86))
+    chunk_us: float = 0.744           # one 256-pattern chunk of a weight tile
+    weight_fixed_us: float = 1.35     # chunk issue, tile reduction and update
+    skew_us: float = 0.86             # arrival skew between CTAs, the remainder at B = 512
     # one-CTA kernel: per group of B patterns
-    small_us: tuple = ((1, 6.75), (2, 7.35), (4, 9.16))
+    small_us: tuple = ((1, 6.68), (2, 7.37), (4, 9.17))
 
 
 def gb300_group_size(B, n_sm=152, max_pg=8):
