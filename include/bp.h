@@ -25,6 +25,10 @@
  *   - Patterns are row-major: X is [batch, n_0], T and Y are [batch, n_L].
  *     Their element type is float32 for BP_F32 nets and bfloat16 (raw uint16
  *     bits, round-to-nearest-even) for BP_BF16 nets.  Targets are in [0, 1].
+ *   - Alignment: device pattern buffers (X, T, Y) start on a 16-byte boundary
+ *     for BP_BF16 nets (their rows move in 16-byte pieces) and on a 4-byte
+ *     boundary for BP_F32 nets; error-sum buffers on a 4-byte boundary.  Other
+ *     pointers are rejected with BP_EINVAL before any work is queued.
  *   - Device pointers ("d_") are caller-owned CUDA device memory on the current
  *     device; the library never frees them.  Host pointers ("h_") are caller-
  *     owned host memory (pinned memory makes the copies asynchronous).

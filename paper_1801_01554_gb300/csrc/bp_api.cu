@@ -123,6 +123,20 @@ bp_status check_batch(const bp_net* net, int batch) {
     return BP_OK;
 }
 
+// Pattern and output buffers: the bf16 kernels move rows in 16-byte pieces, the
+// float32 kernels in 4-byte words.  The error sums are float32 words.
+bp_status check_align(const bp_net* net, const void* X, const void* T, const void* Y,
+                      const float* sse) {
+    const uintptr_t a = net->dtype == BP_BF16 ? 16 : 4;
+    const void* p[3] = {X, T, Y};
+    const char* what[3] = {"X", "T", "Y"};
+    for (int k = 0; k < 3; ++k)
+        if (((uintptr_t)p[k] & (a - 1)) != 0)
+            return fail(BP_EINVAL, "%s must be %d-byte aligned for this net's dtype", what[k], (int)a);
+    if (((uintptr_t)sse & 3) != 0) return fail(BP_EINVAL, "the error-sum buffer must be 4-byte aligned");
+    return BP_OK;
+}
+
 }  // namespace
 
 extern "C" {
@@ -305,6 +319,7 @@ bp_status bp_diagnose(bp_net* net, const void* d_X, const void* d_T, int batch, 
         return fail(BP_EINVAL, "NULL argument");
     if (net->dtype != BP_F32) return fail(BP_EINVAL, "the diagnostic mode is implemented for float32 nets");
     bp_status st = check_batch(net, batch);
+    if (st == BP_OK) st = check_align(net, d_X, d_T, nullptr, nullptr);
     if (st != BP_OK) return st;
     const int n = net->num_sms;
     if ((h_sse != nullptr || h_sm != nullptr) && capacity < n)
@@ -378,6 +393,7 @@ bp_status bp_get_grads(const bp_net* net, float* h) {
 bp_status bp_forward(bp_net* net, const void* d_X, int batch, void* d_Y, void* stream) {
     if (net == nullptr || d_X == nullptr) return fail(BP_EINVAL, "NULL argument");
     bp_status st = check_batch(net, batch);
+    if (st == BP_OK) st = check_align(net, d_X, nullptr, d_Y, nullptr);
     if (st != BP_OK) return st;
     cudaStream_t s = (cudaStream_t)stream;
     if (net->dtype == BP_F32) {
@@ -395,6 +411,7 @@ bp_status bp_forward(bp_net* net, const void* d_X, int batch, void* d_Y, void* s
 bp_status bp_backward(bp_net* net, const void* d_T, int batch, float* d_sse, void* stream) {
     if (net == nullptr || d_T == nullptr) return fail(BP_EINVAL, "NULL argument");
     bp_status st = check_batch(net, batch);
+    if (st == BP_OK) st = check_align(net, nullptr, d_T, nullptr, d_sse);
     if (st != BP_OK) return st;
     if (net->fwd_batch == 0) return fail(BP_ESTATE, "bp_backward needs a preceding bp_forward");
     if (net->fwd_batch != batch)
@@ -453,6 +470,7 @@ bp_status bp_train_batch(bp_net* net, const void* d_X, const void* d_T, int batc
                          void* stream) {
     if (net == nullptr || d_X == nullptr || d_T == nullptr) return fail(BP_EINVAL, "NULL argument");
     bp_status st = check_batch(net, batch);
+    if (st == BP_OK) st = check_align(net, d_X, d_T, nullptr, d_sse);
     if (st != BP_OK) return st;
     return run_epoch(net, d_X, d_T, batch, batch, d_sse, (cudaStream_t)stream);
 }
@@ -462,6 +480,7 @@ bp_status bp_train_epoch(bp_net* net, const void* d_X, const void* d_T, int n_pa
     if (net == nullptr || d_X == nullptr || d_T == nullptr) return fail(BP_EINVAL, "NULL argument");
     if (n_patterns < 1) return fail(BP_EINVAL, "n_patterns must be >= 1 (got %d)", n_patterns);
     bp_status st = check_batch(net, minibatch);
+    if (st == BP_OK) st = check_align(net, d_X, d_T, nullptr, d_sse);
     if (st != BP_OK) return st;
     return run_epoch(net, d_X, d_T, n_patterns, minibatch, d_sse, (cudaStream_t)stream);
 }

@@ -216,15 +216,6 @@ __device__ __forceinline__ void reduce_scatter32(float (&v)[32], int lane) {
 __device__ __forceinline__ void epi_bar() { asm volatile("bar.sync 1, 128;" ::: "memory"); }
 
 // ------------------------------------------------------------ epilogue
-__device__ __forceinline__ void tma_store_2d(const CUtensorMap* map, const void* smem_src, int c0,
-                                             int c1) {
-    asm volatile(
-        "cp.async.bulk.tensor.2d.global.shared::cta.bulk_group [%0, {%1, %2}], [%3];" ::"l"(
-            (unsigned long long)map),
-        "r"(c0), "r"(c1), "r"(smem_u32(smem_src))
-        : "memory");
-}
-
 // 32 consecutive bf16 of one row as floats (16-byte loads when the row segment is whole).
 __device__ __forceinline__ void load_row32(float (&a)[32], const bf16* p, bool whole, int valid) {
     if (whole) {
@@ -246,14 +237,16 @@ __device__ __forceinline__ void load_row32(float (&a)[32], const bf16* p, bool w
 }
 
 // One 32-column chunk of the tile for the 32 rows of one epilogue warp (this
-// lane's row m).  Values are rounded to bf16, staged per warp in shared memory
-// (sR: the rows, sT: the same block transposed) and written by TMA stores; the
-// column sums of a delta block (bias change) are read back from sT.
+// lane's row m).  Values are rounded to bf16 and staged per warp in shared
+// memory (sR: the 32 x 32 block by rows, its 16-byte pieces permuted by row so
+// that the lanes' writes hit distinct banks; sT: the block transposed).  The
+// warp then writes each 64-byte row (or column) segment with four lanes'
+// 16-byte stores, eight segments per instruction.  The column sums of a delta
+// block (bias change) are read back from sT.
 template <int MODE>
-__device__ __forceinline__ void epilogue_chunk(const GemmArgs& g, const CUtensorMap* map_r,
-                                               const CUtensorMap* map_t, int m, int m0, int n0,
-                                               int split, float (&v)[32], float& sse, bool row_ok,
-                                               bf16* sR, bf16* sT, float* colsum_slot) {
+__device__ __forceinline__ void epilogue_chunk(const GemmArgs& g, int m, int m0, int n0, int split,
+                                               float (&v)[32], float& sse, bool row_ok, bf16* sR,
+                                               bf16* sT, float* colsum_slot) {
     const int N = g.N;
     const int lane = threadIdx.x & 31;
     if (MODE == MODE_DW) {
@@ -312,29 +305,56 @@ __device__ __forceinline__ void epilogue_chunk(const GemmArgs& g, const CUtensor
             vals[c] = ok ? bf16_round(v[c] * a[c] * (1.f - a[c])) : 0.f;
         }
     }
-    const bool has_r = (MODE == MODE_FWD) || (MODE == MODE_FWD_OUT) ||
-                       (MODE == MODE_DX && g.out != nullptr);
+    // rows: A_l, A_L or delta_L (training output layer), or delta_{l-1}
+    bf16* const rows = with_t ? g.out2 : g.out;
+    const int ldr = with_t ? g.ld2 : g.ldo;
+    const bool has_r = rows != nullptr;
     const bool has_t = (MODE == MODE_FWD && g.out_t != nullptr) || with_t || (MODE == MODE_DX);
+    uint4* sR4 = reinterpret_cast<uint4*>(sR);
     if (has_r) {
-        uint4* dst = reinterpret_cast<uint4*>(sR + lane * 32);
 #pragma unroll
         for (int k = 0; k < 4; ++k) {
             __align__(16) __nv_bfloat162 h[4];
 #pragma unroll
             for (int q = 0; q < 4; ++q) h[q] = __floats2bfloat162_rn(vals[8 * k + 2 * q], vals[8 * k + 2 * q + 1]);
-            dst[k] = *reinterpret_cast<const uint4*>(h);
+            sR4[lane * 4 + (k ^ ((lane >> 1) & 3))] = *reinterpret_cast<const uint4*>(h);
         }
     }
     if (has_t) {
 #pragma unroll
         for (int c = 0; c < 32; ++c) sT[c * 32 + lane] = __float2bfloat16_rn(vals[c]);
     }
-    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
     __syncwarp();
-    if (lane == 0) {
-        if (has_r) tma_store_2d(map_r, sR, n0, m0);
-        if (has_t) tma_store_2d(map_t, sT, m0, n0);
-        asm volatile("cp.async.bulk.commit_group;" ::: "memory");
+    const int piece = lane & 3;   // 16-byte piece of a 64-byte segment
+    if (has_r) {
+        const int pieces = valid >> 3;   // N is a multiple of 8
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+            const int r = j * 8 + (lane >> 2);
+            if (m0 + r < g.M && piece < pieces)
+                *reinterpret_cast<uint4*>(rows + (size_t)(m0 + r) * ldr + n0 + piece * 8) =
+                    sR4[r * 4 + (piece ^ ((r >> 1) & 3))];
+        }
+    }
+    if (has_t) {
+        const uint4* sT4 = reinterpret_cast<const uint4*>(sT);
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+            const int c = j * 8 + (lane >> 2);
+            const int left = g.M - (m0 + piece * 8);   // rows of this piece inside the batch
+            if (c < valid && left > 0) {
+                const uint4 u = sT4[c * 4 + piece];
+                bf16* dst = g.out_t + (size_t)(n0 + c) * g.ldt + m0 + piece * 8;
+                if (left >= 8) {
+                    *reinterpret_cast<uint4*>(dst) = u;
+                } else {
+                    const bf16* e = reinterpret_cast<const bf16*>(&u);
+#pragma unroll
+                    for (int i = 0; i < 8; ++i)
+                        if (i < left) dst[i] = e[i];
+                }
+            }
+        }
     }
     if (colsum_slot != nullptr) {
         // lane c sums column c of the block over the warp's 32 rows
@@ -353,7 +373,6 @@ __device__ __forceinline__ void epilogue_chunk(const GemmArgs& g, const CUtensor
         }
         colsum_slot[lane] = sum;
     }
-    if (lane == 0) asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory");
     __syncwarp();   // the staging blocks may be rewritten
 }
 
@@ -375,7 +394,6 @@ struct GemmCfg {
 template <int BN, int MODE>
 __global__ void __launch_bounds__(kGemmThreads, 1)
     k_gemm(const __grid_constant__ CUtensorMap map_a, const __grid_constant__ CUtensorMap map_b,
-           const __grid_constant__ CUtensorMap map_r, const __grid_constant__ CUtensorMap map_t,
            GemmArgs g) {
     using Cfg = GemmCfg<BN, MODE>;
     constexpr int S = Cfg::kStages;
@@ -531,7 +549,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
                     if (want_colsum) colsum[ew * BN + c0 + lane] = 0.f;
                     continue;
                 }
-                epilogue_chunk<MODE>(g, &map_r, &map_t, m, m0, n0, split, v, sse, row_ok, sR, sT,
+                epilogue_chunk<MODE>(g, m, m0, n0, split, v, sse, row_ok, sR, sT,
                                      want_colsum ? colsum + ew * BN + c0 : nullptr);
             }
             // TMEM is free for the next accumulation into this buffer
@@ -562,7 +580,6 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
             }
         }
     }
-    if (warp >= 2 && lane == 0) asm volatile("cp.async.bulk.wait_group 0;" ::: "memory");
     tc_fence_before();
     __syncthreads();
     if (warp == 1) {
@@ -800,18 +817,6 @@ bool make_map(CUtensorMap* map, const void* base, int rows, int cols, int ld, in
     return r == CUDA_SUCCESS;
 }
 
-// Store map: [rows, cols] bf16, row pitch ld elements, 32 x 32 boxes, no swizzle.
-bool make_store_map(CUtensorMap* map, const void* base, int rows, int cols, int ld) {
-    cuuint64_t dims[2] = {(cuuint64_t)cols, (cuuint64_t)rows};
-    cuuint64_t strides[1] = {(cuuint64_t)ld * 2};
-    cuuint32_t box[2] = {32, 32};
-    cuuint32_t estr[2] = {1, 1};
-    CUresult r = g_encode(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims,
-                          strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
-                          CU_TENSOR_MAP_SWIZZLE_NONE, CU_TENSOR_MAP_L2_PROMOTION_NONE,
-                          CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
-    return r == CUDA_SUCCESS;
-}
 
 template <int BN, int MODE>
 cudaError_t gemm_setup() {
@@ -883,7 +888,7 @@ int pick_splits(int tiles, int kb_total, int num_sms, int cap_splits) {
 
 template <int MODE>
 cudaError_t launch_gemm(const Bf16Net* b, const CUtensorMap& ma, const CUtensorMap& mb,
-                        const CUtensorMap& mr, const CUtensorMap& mt, GemmArgs g, cudaStream_t s) {
+                        GemmArgs g, cudaStream_t s) {
     g.num_m = ceil_div(g.M, BM);
     g.num_n = ceil_div(g.N, kBN);
     g.kb_total = ceil_div(g.K, BK);
@@ -893,7 +898,7 @@ cudaError_t launch_gemm(const Bf16Net* b, const CUtensorMap& ma, const CUtensorM
     g.flags = b->flags;
     const int items = g.num_m * g.num_n * g.splits;
     const int grid = items < b->num_sms ? items : b->num_sms;
-    k_gemm<kBN, MODE><<<grid, kGemmThreads, GemmCfg<kBN, MODE>::kSmemBytes, s>>>(ma, mb, mr, mt, g);
+    k_gemm<kBN, MODE><<<grid, kGemmThreads, GemmCfg<kBN, MODE>::kSmemBytes, s>>>(ma, mb, g);
     return cudaGetLastError();
 }
 
@@ -919,16 +924,12 @@ cudaError_t run_forward(Bf16Net* b, const bf16* X, int B, const bf16* T, bf16* Y
         g.K = b->n[l - 1];
         g.bias = b->theta + b->boff[l];
         cudaError_t e;
-        CUtensorMap mr, mt;
         if (l < L) {
             g.out = b->act[l];
             g.ldo = b->n[l];
             g.out_t = b->actT[l];
             g.ldt = b->cap_pad;
-            if (!make_store_map(&mr, g.out, B, b->n[l], b->n[l]) ||
-                !make_store_map(&mt, g.out_t, b->n[l], B, b->cap_pad))
-                return cudaErrorInvalidValue;
-            e = launch_gemm<MODE_FWD>(b, ma, mb, mr, mt, g, s);
+            e = launch_gemm<MODE_FWD>(b, ma, mb, g, s);
         } else {
             if (T != nullptr) {
                 // training: the output deltas (rows and transposed) replace the outputs
@@ -940,16 +941,11 @@ cudaError_t run_forward(Bf16Net* b, const bf16* X, int B, const bf16* T, bf16* Y
                 g.ldt = b->cap_pad;
                 g.bias_part = b->bpart[L];
                 g.sse_part = b->sse_part;
-                if (!make_store_map(&mr, g.out2, B, b->n[L], b->n[L]) ||
-                    !make_store_map(&mt, g.out_t, b->n[L], B, b->cap_pad))
-                    return cudaErrorInvalidValue;
             } else {
                 g.out = (Y != nullptr) ? Y : b->act[L];
                 g.ldo = b->n[L];
-                if (!make_store_map(&mr, g.out, B, b->n[L], b->n[L])) return cudaErrorInvalidValue;
-                mt = mr;
             }
-            e = launch_gemm<MODE_FWD_OUT>(b, ma, mb, mr, mt, g, s);
+            e = launch_gemm<MODE_FWD_OUT>(b, ma, mb, g, s);
         }
         if (e != cudaSuccess) return e;
     }
@@ -984,14 +980,7 @@ cudaError_t run_backward(Bf16Net* b, const bf16* X, int B, cudaStream_t s) {
         g.aux = b->act[l - 1];
         g.ld_aux = b->n[l - 1];
         g.bias_part = b->bpart[l - 1];
-        CUtensorMap mr, mt;
-        if (!make_store_map(&mt, g.out_t, b->n[l - 1], B, b->cap_pad)) return cudaErrorInvalidValue;
-        if (g.out != nullptr) {
-            if (!make_store_map(&mr, g.out, B, b->n[l - 1], b->n[l - 1])) return cudaErrorInvalidValue;
-        } else {
-            mr = mt;
-        }
-        cudaError_t e = launch_gemm<MODE_DX>(b, ma, mb, mr, mt, g, s);
+        cudaError_t e = launch_gemm<MODE_DX>(b, ma, mb, g, s);
         if (e != cudaSuccess) return e;
     }
     for (int l = 1; l <= L; ++l) {
@@ -1008,7 +997,7 @@ cudaError_t run_backward(Bf16Net* b, const bf16* X, int B, cudaStream_t s) {
         g.splits = b->splits[l];
         const int tiles = ceil_div(g.M, BM) * ceil_div(g.N, kBN);
         g.splits = pick_splits(tiles, ceil_div(B, BK), b->num_sms, b->splits[l]);
-        cudaError_t e = launch_gemm<MODE_DW>(b, ma, mb, ma, ma, g, s);
+        cudaError_t e = launch_gemm<MODE_DW>(b, ma, mb, g, s);
         if (e != cudaSuccess) return e;
     }
     return cudaSuccess;

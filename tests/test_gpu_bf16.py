@@ -239,3 +239,28 @@ def test_deepest_net_the_boundary_allows():
         net.check()
         assert normwise(Y.float().cpu().numpy(), Y_ref) <= TOL
         assert normwise(net.get_weights() - theta, st.theta - theta) <= TOL
+
+
+def test_misaligned_pattern_buffers_are_rejected_before_any_launch():
+    """bf16 rows move in 16-byte pieces: X, T and Y must start on a 16-byte
+    boundary.  A buffer offset by one element is refused with BP_EINVAL and
+    the net stays usable."""
+    sizes, B = (64, 128, 32), 64
+    X, T, theta = problem(sizes, B, seed=3)
+    Xd = dev_bf16(np.vstack([X, X[:1]])).flatten()
+    Td = dev_bf16(np.vstack([T, T[:1]])).flatten()
+    with bp.Net(sizes, 0.05, 0.9, bp.BP_BF16, max_batch=B) as net:
+        net.set_weights(theta)
+        for args in ((Xd[1:], Td[:B * sizes[-1]]), (Xd[:B * sizes[0]], Td[1:])):
+            with pytest.raises(bp.BPError) as e:
+                net.train_batch(args[0], args[1], B)
+            assert e.value.status == bp.BP_EINVAL
+        Y = torch.empty(B * sizes[-1] + 8, dtype=torch.bfloat16, device="cuda")
+        with pytest.raises(bp.BPError) as e:
+            net.forward(Xd[:B * sizes[0]], B, Y[1:])
+        assert e.value.status == bp.BP_EINVAL
+        net.train_batch(Xd[:B * sizes[0]], Td[:B * sizes[-1]], B)
+        net.check()
+        st = O.State(sizes, theta, lr=0.05, momentum=0.9)
+        O.train_batch(st, X, T)
+        assert normwise(net.get_weights() - theta, st.theta - theta) <= TOL

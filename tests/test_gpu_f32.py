@@ -437,6 +437,13 @@ def test_argument_and_state_errors():
         with pytest.raises(bp.BPError) as e:
             net.set_hparams(float("nan"), 0.9)
         assert e.value.status == bp.BP_EINVAL
+        # float32 rows are read word by word: a buffer off a 4-byte boundary is refused
+        with pytest.raises(bp.BPError) as e:
+            net.train_batch(X.data_ptr() + 2, T, 8)
+        assert e.value.status == bp.BP_EINVAL
+        with pytest.raises(bp.BPError) as e:
+            net.train_batch(X, T, 8, T.data_ptr() + 1)
+        assert e.value.status == bp.BP_EINVAL
         net.check()
 
 
