@@ -44,8 +44,9 @@ using bf16 = __nv_bfloat16;
 constexpr int BM = 128;   // rows of a tile (TMEM lanes)
 constexpr int BK = 64;    // K per stage: 64 bf16 = one 128-byte swizzle row
 constexpr int UMMA_K = 16;
-constexpr int kGemmThreads = 192;   // warp 0 TMA, warp 1 MMA, warps 2..5 epilogue
-constexpr int kEpiThreads = 128;
+constexpr int kEpiWarps = 8;         // two per TMEM lane quarter, each on half of the columns
+constexpr int kEpiThreads = 32 * kEpiWarps;
+constexpr int kGemmThreads = 64 + kEpiThreads;   // warp 0 TMA, warp 1 MMA, warps 2.. epilogue
 
 constexpr unsigned long long kWaitNs = 2000000000ull;
 constexpr unsigned kWaitIters = 1u << 28;
@@ -213,7 +214,7 @@ __device__ __forceinline__ void reduce_scatter32(float (&v)[32], int lane) {
     }
 }
 
-__device__ __forceinline__ void epi_bar() { asm volatile("bar.sync 1, 128;" ::: "memory"); }
+__device__ __forceinline__ void epi_bar() { asm volatile("bar.sync 1, %0;" ::"n"(kEpiThreads) : "memory"); }
 
 // ------------------------------------------------------------ epilogue
 // 32 consecutive bf16 of one row as floats (16-byte loads when the row segment is whole).
@@ -237,16 +238,16 @@ __device__ __forceinline__ void load_row32(float (&a)[32], const bf16* p, bool w
 }
 
 // One 32-column chunk of the tile for the 32 rows of one epilogue warp (this
-// lane's row m).  Values are rounded to bf16 and staged per warp in shared
-// memory (sR: the 32 x 32 block by rows, its 16-byte pieces permuted by row so
-// that the lanes' writes hit distinct banks; sT: the block transposed).  The
-// warp then writes each 64-byte row (or column) segment with four lanes'
+// lane's row m).  Values are rounded to bf16 and staged in the warp's 2 KB
+// shared-memory block, first by rows (16-byte pieces permuted by row so that
+// the lanes' writes hit distinct banks), then transposed.  After each staging
+// the warp writes every 64-byte row (or column) segment with four lanes'
 // 16-byte stores, eight segments per instruction.  The column sums of a delta
-// block (bias change) are read back from sT.
+// block (bias change) are read back from the transposed block.
 template <int MODE>
 __device__ __forceinline__ void epilogue_chunk(const GemmArgs& g, int m, int m0, int n0, int split,
-                                               float (&v)[32], float& sse, bool row_ok, bf16* sR,
-                                               bf16* sT, float* colsum_slot) {
+                                               float (&v)[32], float& sse, bool row_ok, bf16* sS,
+                                               const float* sbias, float* colsum_slot) {
     const int N = g.N;
     const int lane = threadIdx.x & 31;
     if (MODE == MODE_DW) {
@@ -268,19 +269,14 @@ __device__ __forceinline__ void epilogue_chunk(const GemmArgs& g, int m, int m0,
     const bool with_t = (MODE == MODE_FWD_OUT) && (g.aux != nullptr);
     float vals[32];
     if (MODE == MODE_FWD || MODE == MODE_FWD_OUT) {
-        float b[32];
-        if (whole) {
+        float b[32];   // the tile's biases, staged in shared memory (0 past N)
 #pragma unroll
-            for (int k = 0; k < 8; ++k) {
-                const float4 f = __ldg(reinterpret_cast<const float4*>(g.bias + n0) + k);
-                b[4 * k] = f.x;
-                b[4 * k + 1] = f.y;
-                b[4 * k + 2] = f.z;
-                b[4 * k + 3] = f.w;
-            }
-        } else {
-#pragma unroll
-            for (int c = 0; c < 32; ++c) b[c] = (c < valid) ? __ldg(g.bias + n0 + c) : 0.f;
+        for (int k = 0; k < 8; ++k) {
+            const float4 f = reinterpret_cast<const float4*>(sbias)[k];
+            b[4 * k] = f.x;
+            b[4 * k + 1] = f.y;
+            b[4 * k + 2] = f.z;
+            b[4 * k + 3] = f.w;
         }
         float t[32];
         if (with_t) load_row32(t, g.aux + (size_t)m * g.ld_aux + n0, whole && row_ok, row_ok ? valid : 0);
@@ -310,40 +306,37 @@ __device__ __forceinline__ void epilogue_chunk(const GemmArgs& g, int m, int m0,
     const int ldr = with_t ? g.ld2 : g.ldo;
     const bool has_r = rows != nullptr;
     const bool has_t = (MODE == MODE_FWD && g.out_t != nullptr) || with_t || (MODE == MODE_DX);
-    uint4* sR4 = reinterpret_cast<uint4*>(sR);
+    uint4* sS4 = reinterpret_cast<uint4*>(sS);
+    const int piece = lane & 3;   // 16-byte piece of a 64-byte segment
     if (has_r) {
 #pragma unroll
         for (int k = 0; k < 4; ++k) {
             __align__(16) __nv_bfloat162 h[4];
 #pragma unroll
             for (int q = 0; q < 4; ++q) h[q] = __floats2bfloat162_rn(vals[8 * k + 2 * q], vals[8 * k + 2 * q + 1]);
-            sR4[lane * 4 + (k ^ ((lane >> 1) & 3))] = *reinterpret_cast<const uint4*>(h);
+            sS4[lane * 4 + (k ^ ((lane >> 1) & 3))] = *reinterpret_cast<const uint4*>(h);
         }
-    }
-    if (has_t) {
-#pragma unroll
-        for (int c = 0; c < 32; ++c) sT[c * 32 + lane] = __float2bfloat16_rn(vals[c]);
-    }
-    __syncwarp();
-    const int piece = lane & 3;   // 16-byte piece of a 64-byte segment
-    if (has_r) {
+        __syncwarp();
         const int pieces = valid >> 3;   // N is a multiple of 8
 #pragma unroll
         for (int j = 0; j < 4; ++j) {
             const int r = j * 8 + (lane >> 2);
             if (m0 + r < g.M && piece < pieces)
                 *reinterpret_cast<uint4*>(rows + (size_t)(m0 + r) * ldr + n0 + piece * 8) =
-                    sR4[r * 4 + (piece ^ ((r >> 1) & 3))];
+                    sS4[r * 4 + (piece ^ ((r >> 1) & 3))];
         }
+        __syncwarp();   // the block is rewritten below
     }
     if (has_t) {
-        const uint4* sT4 = reinterpret_cast<const uint4*>(sT);
+#pragma unroll
+        for (int c = 0; c < 32; ++c) sS[c * 32 + lane] = __float2bfloat16_rn(vals[c]);
+        __syncwarp();
 #pragma unroll
         for (int j = 0; j < 4; ++j) {
             const int c = j * 8 + (lane >> 2);
             const int left = g.M - (m0 + piece * 8);   // rows of this piece inside the batch
             if (c < valid && left > 0) {
-                const uint4 u = sT4[c * 4 + piece];
+                const uint4 u = sS4[c * 4 + piece];
                 bf16* dst = g.out_t + (size_t)(n0 + c) * g.ldt + m0 + piece * 8;
                 if (left >= 8) {
                     *reinterpret_cast<uint4*>(dst) = u;
@@ -358,7 +351,7 @@ __device__ __forceinline__ void epilogue_chunk(const GemmArgs& g, int m, int m0,
     }
     if (colsum_slot != nullptr) {
         // lane c sums column c of the block over the warp's 32 rows
-        const uint4* col = reinterpret_cast<const uint4*>(sT + lane * 32);
+        const uint4* col = reinterpret_cast<const uint4*>(sS + lane * 32);
         float sum = 0.f;
 #pragma unroll
         for (int k = 0; k < 4; ++k) {
@@ -387,8 +380,10 @@ struct GemmCfg {
     // tile ring, then barriers and scratch
     static constexpr int kRingBytes = kStages * kStageBytes;
     static constexpr int kColsumBytes = 4 * BN * 4;
-    static constexpr int kStageOutBytes = 4 * 2 * 32 * 32 * 2;   // per epilogue warp: rows + transposed
-    static constexpr int kSmemBytes = 1024 + kRingBytes + kColsumBytes + kStageOutBytes + 256;
+    static constexpr int kStageOutBytes = kEpiWarps * 32 * 32 * 2;   // one 32 x 32 bf16 block per epilogue warp
+    static constexpr int kBiasBytes = 2 * BN * 4;   // the tile's biases, one block per accumulator
+    static constexpr int kSmemBytes =
+        1024 + kRingBytes + kColsumBytes + kStageOutBytes + kBiasBytes + 256;
 };
 
 template <int BN, int MODE>
@@ -402,8 +397,10 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
     uint8_t* ring = smem;
     float* colsum = reinterpret_cast<float*>(smem + Cfg::kRingBytes);   // [4][BN]
     bf16* stage_out = reinterpret_cast<bf16*>(smem + Cfg::kRingBytes + Cfg::kColsumBytes);
+    float* bias_s = reinterpret_cast<float*>(smem + Cfg::kRingBytes + Cfg::kColsumBytes +
+                                             Cfg::kStageOutBytes);   // [2][BN]
     uint64_t* bars = reinterpret_cast<uint64_t*>(smem + Cfg::kRingBytes + Cfg::kColsumBytes +
-                                                 Cfg::kStageOutBytes);
+                                                 Cfg::kStageOutBytes + Cfg::kBiasBytes);
     uint64_t* full = bars;              // [S]
     uint64_t* empty = bars + S;         // [S]
     uint64_t* tfull = bars + 2 * S;     // [2]
@@ -521,16 +518,26 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
             }
         }
     } else {
-        // ---------------- epilogue warps 2..5
+        // ---------------- epilogue warps 2..9
         const int q = warp & 3;                  // TMEM lane quarter this warp may access
-        const int ew = warp - 2;                 // 0..3 slot in the column-sum scratch
+        const int ew = warp - 2;                 // 0..7
+        const int slot = ew & 3;                 // row quarter's slot in the column-sum scratch
+        const int cbeg = (ew >> 2) * (BN / 2);   // this warp's half of the columns
         int acc = 0;
         unsigned acc_phase = 0;
         for (int it = blockIdx.x; it < items; it += gridDim.x) {
             const int tile = it % tiles, split = it / tiles;
             const int mb = tile % g.num_m, nb = tile / g.num_m;
+            float* sbias = bias_s + acc * BN;
+            if (MODE == MODE_FWD || MODE == MODE_FWD_OUT) {
+                // block acc was last read two tiles ago, before the barrier of the previous tile
+                for (int c = threadIdx.x - 64; c < BN; c += kEpiThreads) {
+                    const int n = nb * BN + c;
+                    sbias[c] = n < g.N ? __ldg(g.bias + n) : 0.f;
+                }
+            }
             mbar_wait(&tfull[acc], acc_phase, abort_flag, g.flags);
-            epi_bar();                     // the four warps leave together on an abort
+            epi_bar();                     // the epilogue warps leave together on an abort
             if (*abort_flag) break;
             tc_fence_after();
             const int m = mb * BM + q * 32 + lane;
@@ -538,19 +545,18 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
             float sse = 0.f;
             const uint32_t tbase = tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(acc * BN);
             const int m0 = mb * BM + q * 32;
-            bf16* sR = stage_out + ew * 2048;
-            bf16* sT = sR + 1024;
+            bf16* sS = stage_out + ew * 1024;
             const bool want_colsum = (MODE == MODE_DX) || (MODE == MODE_FWD_OUT && g.aux != nullptr);
-            for (int c0 = 0; c0 < BN; c0 += 32) {
+            for (int c0 = cbeg; c0 < cbeg + BN / 2; c0 += 32) {
                 const int n0 = nb * BN + c0;
                 float v[32];
                 tmem_ld32(tbase + (uint32_t)c0, v);
                 if (n0 >= g.N) {
-                    if (want_colsum) colsum[ew * BN + c0 + lane] = 0.f;
+                    if (want_colsum) colsum[slot * BN + c0 + lane] = 0.f;
                     continue;
                 }
-                epilogue_chunk<MODE>(g, m, m0, n0, split, v, sse, row_ok, sR, sT,
-                                     want_colsum ? colsum + ew * BN + c0 : nullptr);
+                epilogue_chunk<MODE>(g, m, m0, n0, split, v, sse, row_ok, sS, sbias + c0,
+                                     want_colsum ? colsum + slot * BN + c0 : nullptr);
             }
             // TMEM is free for the next accumulation into this buffer
             tc_fence_before();
@@ -558,7 +564,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
             if (++acc == 2) { acc = 0; acc_phase ^= 1u; }
             if (MODE == MODE_DX || (MODE == MODE_FWD_OUT && g.aux != nullptr)) {
                 epi_bar();
-                const int t = threadIdx.x - 64;   // 0..127
+                const int t = threadIdx.x - 64;   // 0 .. kEpiThreads - 1
                 for (int c = t; c < BN; c += kEpiThreads) {
                     const int n = nb * BN + c;
                     if (n < g.N) {
@@ -567,14 +573,15 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
                     }
                 }
                 if (MODE == MODE_FWD_OUT) {
-                    // tile error sum: warp sums, then the four warps in a fixed order
+                    // tile error sum: warp sums, then the eight warps in a fixed order
 #pragma unroll
                     for (int o = 16; o > 0; o >>= 1) sse += __shfl_xor_sync(0xffffffffu, sse, o);
                     epi_bar();
                     if (lane == 0) colsum[ew] = sse;
                     epi_bar();
                     if (t == 0)
-                        g.sse_part[tile] = (colsum[0] + colsum[1]) + (colsum[2] + colsum[3]);
+                        g.sse_part[tile] = ((colsum[0] + colsum[1]) + (colsum[2] + colsum[3])) +
+                                           ((colsum[4] + colsum[5]) + (colsum[6] + colsum[7]));
                 }
                 epi_bar();
             }
