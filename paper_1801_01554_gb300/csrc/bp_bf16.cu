@@ -658,6 +658,8 @@ __global__ void k_output_delta(const bf16* __restrict__ O, const bf16* __restric
     if (threadIdx.x == 0) sse_part[(size_t)mb * num_n_chunks + nc] = (ss[0] + ss[1]) + (ss[2] + ss[3]);
 }
 
+constexpr int kUT = 64;   // update kernel: weight tile edge
+
 struct LayerUpd {
     int n_out, n_in;
     long long woff, boff;       // offsets in theta / V / G
@@ -671,7 +673,7 @@ struct LayerUpd {
 struct UpdArgs {
     int L;
     LayerUpd ly[kMaxL];
-    int tile0[kMaxL + 1];       // 32x32 weight tiles (+ one bias row band) per layer
+    int tile0[kMaxL + 1];       // kUT x kUT weight tiles (+ one bias row band) per layer
     float* theta;
     float* V;
     float* G;
@@ -696,11 +698,10 @@ __device__ __forceinline__ float guard_change(const UpdArgs& a, float g) {
     return g;
 }
 
-// Momentum update of Section 6.2.1 over 32x32 weight tiles plus the biases:
+// Momentum update of Section 6.2.1 over 64 x 64 weight tiles plus the biases:
 // g = sum of partial changes (+ pending G); v = lr*gs*g + m*v; w += v; then the
 // bf16 copy and its transpose.  Mode 1 adds the partial changes into G instead.
 __global__ void __launch_bounds__(256) k_update_bf16(UpdArgs a) {
-    __shared__ bf16 tileT[32][34];
     if (blockIdx.x == 0 && threadIdx.x == 0 && a.sse_out != nullptr) {
         float s = 0.f;
         for (int k = 0; k < a.n_sse; ++k) s += a.sse_part[k];
@@ -713,70 +714,96 @@ __global__ void __launch_bounds__(256) k_update_bf16(UpdArgs a) {
         while (t >= a.tile0[l + 1]) ++l;
         const LayerUpd& u = a.ly[l];
         const int lt = t - a.tile0[l];
-        const int cols = (u.n_in + 31) / 32;
-        const int rb = lt / cols, cb = lt - rb * cols;   // rb == rows/32 band: biases
-        const int tx = threadIdx.x & 31, ty = threadIdx.x >> 5;
-        const int rows_w = (u.n_out + 31) / 32;
+        const int cols = (u.n_in + kUT - 1) / kUT;
+        const int rb = lt / cols, cb = lt - rb * cols;   // rb == row-tile count: the biases
+        const int rows_w = (u.n_out + kUT - 1) / kUT;
         if (rb < rows_w) {
-            // each thread: column i of rows j = rb*32 + ty + 8r (r < 4); every load of
-            // the four rows is issued before any store
-            const int i = cb * 32 + tx;
-            const float* __restrict__ gp = u.gpart;
-            float* __restrict__ th = a.theta;
-            float* __restrict__ vv = a.V;
-            float* __restrict__ gg = a.G;
-            float gsum[4], w0[4], v0[4], gpend[4];
-            bool ok[4];
-            size_t e[4];
+            // Warp w covers rows 16*(w/2) .. +16 and columns 32*(w%2) .. +32 of the
+            // tile; a lane holds 4 consecutive rows x 4 consecutive columns, so the
+            // fp32 rows move as float4 (8 lanes: one 128-byte line per row) and
+            // both bf16 copies as 8-byte pieces (the transposed copy's 4 rows are
+            // the lane's own).  Layer sizes are multiples of 8: a lane's 4 x 4
+            // block is either inside the layer or outside it.  All loads of the
+            // lane come before its stores.
+            const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
+            const int i = cb * kUT + (w & 1) * 32 + (lane & 7) * 4;
+            const int j0 = rb * kUT + (w >> 1) * 16 + (lane >> 3) * 4;
+            if (i < u.n_in && j0 < u.n_out) {
+                const float4 z = make_float4(0.f, 0.f, 0.f, 0.f);
+                float4 gs[4], w4[4], v4[4], gp4[4];
+                const size_t e0 = (size_t)j0 * u.n_in + i;
+                const float* th = a.theta + u.woff + e0;
+                float* vv = a.V + u.woff + e0;
+                float* gg = a.G + u.woff + e0;
 #pragma unroll
-            for (int r = 0; r < 4; ++r) {
-                const int j = rb * 32 + ty + 8 * r;
-                ok[r] = j < u.n_out && i < u.n_in;
-                e[r] = ok[r] ? (size_t)j * u.n_in + i : 0;
-                gsum[r] = 0.f;
-                w0[r] = 0.f;
-                v0[r] = 0.f;
-                gpend[r] = 0.f;
-            }
-#pragma unroll
-            for (int r = 0; r < 4; ++r) {
-                if (!ok[r]) continue;
-                const long long idx = u.woff + (long long)e[r];
-                if (a.mode != 2)
-                    for (int s = 0; s < u.splits; ++s) gsum[r] += __ldcs(gp + (size_t)s * u.n_out * u.n_in + e[r]);
-                w0[r] = th[idx];
-                if (a.mode == 0) {
-                    v0[r] = vv[idx];
-                    if (a.fold_g) gpend[r] = gg[idx];
-                }
-            }
-#pragma unroll
-            for (int r = 0; r < 4; ++r) {
-                float wv = 0.f;
-                if (ok[r]) {
-                    const long long idx = u.woff + (long long)e[r];
-                    wv = w0[r];
-                    if (a.mode == 1) {
-                        gg[idx] += gsum[r];
-                    } else if (a.mode == 0) {
-                        if (a.fold_g) gg[idx] = 0.f;
-                        const float vel = a.lr_gs * guard_change(a, gsum[r] + gpend[r]) + a.momentum * v0[r];
-                        vv[idx] = vel;
-                        wv += vel;
-                        th[idx] = wv;
+                for (int r = 0; r < 4; ++r) {
+                    gs[r] = z;
+                    v4[r] = z;
+                    gp4[r] = z;
+                    w4[r] = *reinterpret_cast<const float4*>(th + (size_t)r * u.n_in);
+                    if (a.mode == 0) {
+                        v4[r] = *reinterpret_cast<const float4*>(vv + (size_t)r * u.n_in);
+                        if (a.fold_g) gp4[r] = *reinterpret_cast<const float4*>(gg + (size_t)r * u.n_in);
                     }
-                    if (a.mode != 1) u.wb[e[r]] = __float2bfloat16_rn(wv);
                 }
-                tileT[ty + 8 * r][tx] = __float2bfloat16_rn(wv);
-            }
-            if (a.mode != 1) {
-                __syncthreads();
-                for (int k = ty; k < 32; k += 8) {
-                    const int i = cb * 32 + k, j = rb * 32 + tx;
-                    if (i < u.n_in && j < u.n_out) u.wt[(size_t)i * u.n_out + j] = tileT[tx][k];
+                if (a.mode != 2) {
+                    const size_t plane = (size_t)u.n_out * u.n_in;
+                    for (int s = 0; s < u.splits; ++s) {
+                        const float* gp = u.gpart + s * plane + e0;
+#pragma unroll
+                        for (int r = 0; r < 4; ++r) {
+                            const float4 p = __ldcs(reinterpret_cast<const float4*>(gp + (size_t)r * u.n_in));
+                            gs[r].x += p.x;
+                            gs[r].y += p.y;
+                            gs[r].z += p.z;
+                            gs[r].w += p.w;
+                        }
+                    }
+                }
+#pragma unroll
+                for (int r = 0; r < 4; ++r) {
+                    const size_t o = (size_t)r * u.n_in;
+                    if (a.mode == 1) {
+                        float4 g4 = *reinterpret_cast<const float4*>(gg + o);
+                        g4.x += gs[r].x;
+                        g4.y += gs[r].y;
+                        g4.z += gs[r].z;
+                        g4.w += gs[r].w;
+                        *reinterpret_cast<float4*>(gg + o) = g4;
+                    } else if (a.mode == 0) {
+                        float* wc = &w4[r].x;
+                        float* vc = &v4[r].x;
+                        const float* gc = &gs[r].x;
+                        const float* pc = &gp4[r].x;
+#pragma unroll
+                        for (int c = 0; c < 4; ++c) {
+                            const float vel = a.lr_gs * guard_change(a, gc[c] + pc[c]) + a.momentum * vc[c];
+                            vc[c] = vel;
+                            wc[c] += vel;
+                        }
+                        *reinterpret_cast<float4*>(vv + o) = v4[r];
+                        *reinterpret_cast<float4*>(a.theta + u.woff + e0 + o) = w4[r];
+                        if (a.fold_g) *reinterpret_cast<float4*>(gg + o) = z;
+                    }
+                    if (a.mode != 1) {
+                        __align__(8) __nv_bfloat162 h[2];
+                        h[0] = __floats2bfloat162_rn(w4[r].x, w4[r].y);
+                        h[1] = __floats2bfloat162_rn(w4[r].z, w4[r].w);
+                        *reinterpret_cast<uint2*>(u.wb + e0 + o) = *reinterpret_cast<const uint2*>(h);
+                    }
+                }
+                if (a.mode != 1) {
+                    // W_l^T rows i .. i+3, columns j0 .. j0+3
+#pragma unroll
+                    for (int c = 0; c < 4; ++c) {
+                        __align__(8) __nv_bfloat162 h[2];
+                        h[0] = __floats2bfloat162_rn((&w4[0].x)[c], (&w4[1].x)[c]);
+                        h[1] = __floats2bfloat162_rn((&w4[2].x)[c], (&w4[3].x)[c]);
+                        *reinterpret_cast<uint2*>(u.wt + (size_t)(i + c) * u.n_out + j0) =
+                            *reinterpret_cast<const uint2*>(h);
+                    }
                 }
             }
-            __syncthreads();
         } else if (cb == 0) {
             // biases of this layer
             for (int j = threadIdx.x; j < u.n_out; j += 256) {
@@ -1039,7 +1066,7 @@ UpdArgs upd_args(Bf16Net* b, int B, int mode, bool fold, float lr_gs, float mome
         u.wb = b->wb[l];
         u.wt = b->wt[l];
         a.tile0[l - 1] = tiles;
-        tiles += (ceil_div(u.n_out, 32) + 1) * ceil_div(u.n_in, 32);
+        tiles += (ceil_div(u.n_out, kUT) + 1) * ceil_div(u.n_in, kUT);
     }
     a.tile0[b->L] = tiles;
     a.theta = b->theta;
