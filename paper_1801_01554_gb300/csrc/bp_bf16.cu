@@ -598,20 +598,42 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
 }
 
 // ------------------------------------------------------------ SIMT kernels
-// dst[c][r] = src[r][c] for a [rows, cols] bf16 matrix (32 x 32 tiles).
-__global__ void k_transpose(const bf16* __restrict__ src, int rows, int cols, int lds,
-                            bf16* __restrict__ dst, int ldd) {
-    __shared__ bf16 tile[32][34];
-    const int c0 = blockIdx.x * 32, r0 = blockIdx.y * 32;
-    const int tx = threadIdx.x & 31, ty = threadIdx.x >> 5;   // 32 x 8 threads
-    for (int k = ty; k < 32; k += 8) {
-        const int r = r0 + k, c = c0 + tx;
-        tile[k][tx] = (r < rows && c < cols) ? src[(size_t)r * lds + c] : __float2bfloat16_rn(0.f);
+// dst[c][r] = src[r][c] for a [rows, cols] bf16 matrix whose column count and
+// both pitches are multiples of 8 (64 x 64 tiles, 256 threads).  Rows of src
+// and of dst move in 16-byte pieces; the shared-memory pitch of 33 words keeps
+// the lanes' 4-byte writes conflict-free.
+__global__ void __launch_bounds__(256) k_transpose(const bf16* __restrict__ src, int rows, int cols,
+                                                   int lds, bf16* __restrict__ dst, int ldd) {
+    __shared__ __align__(16) uint32_t tile[64][33];   // [r][pair of columns]
+    const int c0 = blockIdx.x * 64, r0 = blockIdx.y * 64;
+    const int t = threadIdx.x, p = t & 7;
+#pragma unroll
+    for (int h = 0; h < 2; ++h) {
+        const int r = (t >> 3) + 32 * h, c = c0 + p * 8;
+        uint4 u = make_uint4(0u, 0u, 0u, 0u);
+        if (r0 + r < rows && c < cols) u = *reinterpret_cast<const uint4*>(src + (size_t)(r0 + r) * lds + c);
+        tile[r][p * 4] = u.x;
+        tile[r][p * 4 + 1] = u.y;
+        tile[r][p * 4 + 2] = u.z;
+        tile[r][p * 4 + 3] = u.w;
     }
     __syncthreads();
-    for (int k = ty; k < 32; k += 8) {
-        const int c = c0 + k, r = r0 + tx;
-        if (c < cols && r < rows) dst[(size_t)c * ldd + r] = tile[tx][k];
+    const bf16* tb = reinterpret_cast<const bf16*>(&tile[0][0]);   // element (r, c) at r * 66 + c
+#pragma unroll
+    for (int h = 0; h < 2; ++h) {
+        const int c = (t >> 3) + 32 * h, r = p * 8;   // dst row c0 + c, columns r0 + r .. +7
+        if (c0 + c >= cols || r0 + r >= rows) continue;
+        __align__(16) bf16 e[8];
+#pragma unroll
+        for (int k = 0; k < 8; ++k) e[k] = tb[(r + k) * 66 + c];
+        bf16* d = dst + (size_t)(c0 + c) * ldd + r0 + r;
+        if (r0 + r + 8 <= rows) {
+            *reinterpret_cast<uint4*>(d) = *reinterpret_cast<const uint4*>(e);
+        } else {
+#pragma unroll
+            for (int k = 0; k < 8; ++k)
+                if (r0 + r + k < rows) d[k] = e[k];
+        }
     }
 }
 
@@ -992,7 +1014,7 @@ cudaError_t run_backward(Bf16Net* b, const bf16* X, int B, cudaStream_t s) {
     const int L = b->L;
     // X^T for the first layer's pooled change
     {
-        dim3 grid(ceil_div(b->n[0], 32), ceil_div(B, 32));
+        dim3 grid(ceil_div(b->n[0], 64), ceil_div(B, 64));
         k_transpose<<<grid, 256, 0, s>>>(X, B, b->n[0], b->n[0], b->actT[0], b->cap_pad);
         cudaError_t e = cudaGetLastError();
         if (e != cudaSuccess) return e;
