@@ -370,6 +370,21 @@ __device__ __forceinline__ void epilogue_chunk(const GemmArgs& g, int m, int m0,
 }
 
 // ------------------------------------------------------------ GEMM kernel
+// Tile order: groups of kGroupM row blocks, each group swept over all column
+// blocks (row block fastest), so that the tiles in flight on the 152 SMs read
+// 16 row blocks of A and about 10 column blocks of B, which stay in L2, instead
+// of every row block of A at once.
+constexpr int kGroupM = 16;
+__device__ __forceinline__ void tile_coords(int tile, int num_m, int num_n, int& mb, int& nb) {
+    const int per_group = kGroupM * num_n;
+    const int grp = tile / per_group;
+    const int first = grp * kGroupM;
+    const int gm = min(num_m - first, kGroupM);
+    const int local = tile - grp * per_group;
+    mb = first + local % gm;
+    nb = local / gm;
+}
+
 template <int BN, int MODE>
 struct GemmCfg {
     static constexpr int kStages = BN == 256 ? 4 : 6;
@@ -448,7 +463,8 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
             bool ok = true;
             for (int it = blockIdx.x; it < items && ok; it += gridDim.x) {
                 const int tile = it % tiles, split = it / tiles;
-                const int mb = tile % g.num_m, nb = tile / g.num_m;
+                int mb, nb;
+                tile_coords(tile, g.num_m, g.num_n, mb, nb);
                 const int kb0 = split * g.kb_per_split;
                 const int kb1 = min(g.kb_total, kb0 + g.kb_per_split);
                 for (int kb = kb0; kb < kb1; ++kb) {
@@ -527,7 +543,8 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
         unsigned acc_phase = 0;
         for (int it = blockIdx.x; it < items; it += gridDim.x) {
             const int tile = it % tiles, split = it / tiles;
-            const int mb = tile % g.num_m, nb = tile / g.num_m;
+            int mb, nb;
+            tile_coords(tile, g.num_m, g.num_n, mb, nb);
             float* sbias = bias_s + acc * BN;
             if (MODE == MODE_FWD || MODE == MODE_FWD_OUT) {
                 // block acc was last read two tiles ago, before the barrier of the previous tile
