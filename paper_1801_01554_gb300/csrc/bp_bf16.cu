@@ -371,10 +371,11 @@ __device__ __forceinline__ void epilogue_chunk(const GemmArgs& g, int m, int m0,
 
 // ------------------------------------------------------------ GEMM kernel
 // Tile order: groups of kGroupM row blocks, each group swept over all column
-// blocks (row block fastest), so that the tiles in flight on the 152 SMs read
-// 16 row blocks of A and about 10 column blocks of B, which stay in L2, instead
-// of every row block of A at once.
-constexpr int kGroupM = 16;
+// blocks (row block fastest), so that the tiles in flight on the 152 SMs share
+// a few row blocks of A and column blocks of B, which stay in L2, instead of
+// reading every row block of A at once (4, 8, 16 and 32 row blocks measured
+// within 2% of each other; one row block at a time was 10% slower for 4096^5).
+constexpr int kGroupM = 4;
 __device__ __forceinline__ void tile_coords(int tile, int num_m, int num_n, int& mb, int& nb) {
     const int per_group = kGroupM * num_n;
     const int grp = tile / per_group;
