@@ -12,11 +12,13 @@
 //     padded rows [W | b | 0..] and activations with a trailing 1, so a row
 //     product is a unit's net input with its bias; the forward pass sums each
 //     dot product as a binary tree across a lane group (Section 10.3).
-//     Activation and delta rows go to scratch rows aligned to 16 bytes.
+//     Activation and delta rows go to global scratch in column blocks
+//     ([cap][32] activations, [cap][8] deltas).
 //
 //   weight phase (Section 5's "bundle" of weights processed over the whole
 //     group of cases): one CTA per 8 x 32 tile of [W_l | b_l] streams the
-//     group's deltas and activations through shared memory with 2-D TMA loads,
+//     group's deltas and activations through shared memory, two contiguous
+//     bulk copies per chunk of 256 patterns,
 //     sums delta[p,j] a[p,i] over all patterns with 4 x 4 register blocks per
 //     lane and a warp butterfly (Sections 3, 4.1), then either accumulates into
 //     G (bp_backward) or applies the momentum update of Section 6.2.1 at once
