@@ -73,8 +73,13 @@ typedef enum {
                      cores with float32 accumulation; float32 master W, b, V, G */
 } bp_dtype;
 
-/* Create a net.  Weights, V and G start at zero (set them with bp_set_weights).
- * layer_sizes: host array of n_layers ints, each >= 1.
+/* Create a net (Section 6.2: the host program turns a network's topology into
+ * the routines that train it; Section 6.2.1: the update routine takes the
+ * learning rate and momentum).  Weights, V and G start at zero (set them with
+ * bp_set_weights).
+ * layer_sizes: host array of n_layers ints, each >= 1 (n_0 inputs ... n_L
+ * outputs; every layer fully connected to the next, plus the true unit).
+ * lr, momentum: the rates of the update routine (Section 6.2.1), finite.
  * dtype: a bp_dtype.  BP_BF16 needs every n_l to be a multiple of 8 (16-byte
  * rows for the tensor-memory copies); any batch size works.
  * max_batch: the largest group any later call may pass (sizes device scratch).
@@ -83,12 +88,15 @@ typedef enum {
 bp_status bp_create(const int* layer_sizes, int n_layers, float lr, float momentum,
                     int dtype, int max_batch, bp_net** out);
 
-/* Free every device buffer of the net.  NULL-safe.  Synchronises the device. */
+/* Free every device buffer of the net (the counterpart of bp_create, Section
+ * 6.2).  NULL-safe.  Synchronises the device.  Caller buffers are untouched. */
 void bp_destroy(bp_net* net);
 
-/* Learning rate, momentum and the factor applied to G in the update
- * (1 = the paper's pooled sum, 1/B = a mean).  Takes effect for work queued
- * after the call.  Errors: BP_EINVAL if a value is not finite. */
+/* Learning rate, momentum and the factor applied to G in the update routine
+ * of Section 6.2.1 (grad_scale 1 = the pooled sum of Sections 3 and 4.1,
+ * 1/B = a mean).  No device work; the net is not touched on failure.  Takes
+ * effect for work queued after the call.  Errors: BP_EINVAL if a value is not
+ * finite. */
 bp_status bp_set_hparams(bp_net* net, float lr, float momentum, float grad_scale);
 
 /* Squashing function of the forward pass (Section 4.3, Figure 3).
@@ -137,13 +145,19 @@ bp_status bp_diagnose(bp_net* net, const void* d_X, const void* d_T, int batch, 
  * and its count to *n_agree.  Host only.  Errors: BP_EINVAL. */
 bp_status bp_vote(const float* values, int n, float* mode, int* n_agree);
 
-/* Number of float32 values in a parameter vector (W and b of every layer). */
+/* Number of float32 values in a parameter vector (W and b of every layer): the
+ * connection count W of Section 7.1, bias connections included (13,826 for
+ * 203-60-26, as Section 6.3 prints).  0 for a NULL net. */
 int64_t bp_num_params(const bp_net* net);
 
 /* Synchronous copies between host float32 arrays of bp_num_params() values and
  * the net's weights (theta), previous weight change (V) or pending pooled
- * change (G).  They synchronise the device first.  bp_set_weights also
- * refreshes the bfloat16 weight copies of a BP_BF16 net. */
+ * change (G) -- the in-memory copies of the weights that Section 10.4 keeps
+ * for checkpoint and recovery; V is the momentum term of Section 6.2.1 and G
+ * the pooled change of Sections 3 and 4.1.  Layout: the packed parameter
+ * vector above.  h_* are caller-owned host arrays, read or written in full.
+ * They synchronise the device first.  bp_set_weights also refreshes the
+ * bfloat16 weight copies of a BP_BF16 net.  Errors: BP_EINVAL (NULL), BP_ECUDA. */
 bp_status bp_set_weights(bp_net* net, const float* h_theta);
 bp_status bp_get_weights(const bp_net* net, float* h_theta);
 bp_status bp_set_velocity(bp_net* net, const float* h_v);
@@ -168,18 +182,25 @@ bp_status bp_backward(bp_net* net, const void* d_T, int batch, float* d_sse, voi
  * W <- W + V; G <- 0 (Section 6.2.1). */
 bp_status bp_update(bp_net* net, void* stream);
 
-/* One whole training step on one group: forward, backward, pooled change and
- * update, with any change already pending in G folded in.  Same buffers and
- * errors as bp_forward + bp_backward. */
+/* One whole training step on one group (Section 3's step with the pooled
+ * change of Section 4.1 and the update of Section 6.2.1): forward, backward,
+ * pooled change over the `batch` patterns and update, with any change already
+ * pending in G folded in.  d_X [batch, n_0], d_T [batch, n_L] caller-owned
+ * device buffers; d_sse NULL or one float (the group's summed squared error).
+ * Errors: BP_EINVAL (NULL, batch out of [1, max_batch], misaligned buffers),
+ * BP_ECUDA; kernel-side errors through bp_check. */
 bp_status bp_train_batch(bp_net* net, const void* d_X, const void* d_T, int batch,
                          float* d_sse, void* stream);
 
 /* One pass over n_patterns patterns taken in index order, one update per
- * minibatch (a ragged last minibatch is a group of its own).  A BP_F32 net runs
- * the whole pass as one persistent device launch; a BP_BF16 net queues one
- * chain of tensor-core kernels per minibatch.  d_sse (may be NULL) receives ceil(n_patterns /
- * minibatch) floats, the error sum of each group.  minibatch <= max_batch.
- * Errors: BP_EINVAL, BP_ECUDA. */
+ * minibatch (Section 3: changes pooled over a group of cases, then applied; a
+ * group of 1 is the per-pattern update, and a ragged last minibatch is a group
+ * of its own).  A BP_F32 net runs the whole pass as one persistent device
+ * launch; a BP_BF16 net queues one chain of tensor-core kernels per minibatch.
+ * d_X [n_patterns, n_0], d_T [n_patterns, n_L] caller-owned device buffers;
+ * d_sse (may be NULL) receives ceil(n_patterns / minibatch) floats, the error
+ * sum of each group.  minibatch <= max_batch.
+ * Errors: BP_EINVAL, BP_ECUDA; kernel-side errors through bp_check. */
 bp_status bp_train_epoch(bp_net* net, const void* d_X, const void* d_T, int n_patterns,
                          int minibatch, float* d_sse, void* stream);
 
@@ -195,9 +216,14 @@ bp_status bp_train_epoch(bp_net* net, const void* d_X, const void* d_T, int n_pa
 bp_status bp_train_epoch_host(bp_net* net, const void* h_X, const void* h_T, int n_patterns,
                               int minibatch, float* h_sse, void* stream);
 
-/* Wait for `stream`, then report and clear errors latched by earlier kernels:
- * BP_ETIMEOUT if a bounded wait ran out, BP_ENONFINITE if an error sum was not
- * finite, else BP_OK (or BP_ECUDA for an error from the CUDA runtime). */
+/* Wait for `stream`, then report and clear errors latched by earlier kernels
+ * (the checks of Section 8: the host learns of a processor's failure and of an
+ * error measure out of range before it trusts the weights):
+ * BP_ETIMEOUT if a bounded wait ran out (the launch stopped early; its updates
+ * so far stand and the grid barrier is reset for the next launch),
+ * BP_ENONFINITE if an error sum was not finite, BP_ESTATE if a check of the
+ * checked build failed, else BP_OK (or BP_ECUDA for an error from the CUDA
+ * runtime).  After it returns, the latch is clear and the net usable. */
 bp_status bp_check(bp_net* net, void* stream);
 
 /* bp_train_epoch for callers that cannot allocate device memory.  The paper
@@ -227,14 +253,32 @@ bp_status bp_check(bp_net* net, void* stream);
  *   calls on a device share the array and find the previous call's contents:
  *   the call clears what must start at zero, and calls that overlap on the GPU
  *   (different streams, or several host threads) race on it.
- *   Asynchronous with respect to the host like bp_train_epoch.  Errors:
- *   BP_EINVAL, BP_ESHAPE, BP_ECUDA. */
+ *   Every minibatch size runs on the grid-wide persistent kernel (152 CTAs and
+ *   two grid barriers per group), including groups of 1-4 patterns, which
+ *   bp_train_epoch sends to its one-CTA kernel.
+ *   Asynchronous with respect to the host like bp_train_epoch.  Pointers are
+ *   checked before any CUDA call: d_theta, d_V, d_X, d_T, d_sse and d_status
+ *   must be 4-byte aligned.  Errors: BP_EINVAL, BP_ESHAPE, BP_ECUDA. */
 bp_status bp_train_epoch_noalloc(const int* layer_sizes, int n_layers, float lr, float momentum,
                                  float grad_scale, float* d_theta, float* d_V, const float* d_X,
                                  const float* d_T, int n_patterns, int minibatch, float* d_sse,
                                  int* d_status, void* stream);
 
-/* Message describing the last failure on the calling thread ("" if none). */
+/* Test hook for the failure detection of Section 8 (a processor that stops
+ * answering must be noticed, not waited for): float32 nets, checked builds
+ * (-DBP_CHECK) only.  Sets the limit of the training kernel's grid-barrier
+ * waits to wait_ns nanoseconds (0 restores the default of 2 s) and, if
+ * unreachable != 0, moves the count that the next training launch's barriers
+ * wait for out of reach, so that its first grid barrier runs out of time: the
+ * launch then latches the timeout, every CTA returns with no copy in flight
+ * and no update applied, and bp_check reports BP_ETIMEOUT and resets the
+ * barrier.  Synchronises the device.  Errors: BP_EINVAL (NULL, a BP_BF16 net),
+ * BP_ESTATE (a library built without BP_CHECK: the hook does nothing there),
+ * BP_ECUDA. */
+bp_status bp_debug_wait_test(bp_net* net, unsigned long long wait_ns, int unreachable);
+
+/* Message describing the last failure on the calling thread ("" if none).
+ * The pointer stays valid until the thread's next call into the library. */
 const char* bp_last_error(void);
 
 #ifdef __cplusplus

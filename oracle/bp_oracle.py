@@ -28,7 +28,7 @@ CMU-CS-89-208):
 * optionally, the fault guard of Section 8: a total weight change outside a
   reasonable range is set to zero and counted before the update.
 
-Readings taken where the paper is silent (each is listed in the design doc):
+Readings taken where the paper is silent:
 
 * the update is the classic momentum rule of the paper's back-propagation
   reference: V <- lr*grad_scale*G + momentum*V, W <- W + V, G <- 0, with V

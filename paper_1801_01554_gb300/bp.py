@@ -52,6 +52,7 @@ SIGNATURES = {
     "bp_check": (_I, [_VP, _VP]),
     "bp_train_epoch_noalloc": (_I, [ctypes.POINTER(_I), _I, _F, _F, _F, _VP, _VP, _VP, _VP, _I, _I,
                                     _VP, _VP, _VP]),
+    "bp_debug_wait_test": (_I, [_VP, ctypes.c_ulonglong, _I]),
     "bp_last_error": (ctypes.c_char_p, []),
 }
 
@@ -265,6 +266,12 @@ def bp_train_epoch_noalloc(sizes, lr, momentum, grad_scale, theta, V, X, T, n_pa
                                          float(grad_scale), _dptr(theta), _dptr(V), _dptr(X),
                                          _dptr(T), int(n_patterns), int(minibatch), _dptr(sse),
                                          _dptr(status), _stream(stream)))
+
+
+def bp_debug_wait_test(h, wait_ns, unreachable):
+    """Checked builds only: grid-barrier wait limit (0 = default) and, with
+    unreachable, a first barrier that the next training launch cannot pass."""
+    _check(load().bp_debug_wait_test(h, int(wait_ns), 1 if unreachable else 0))
 
 
 def bp_last_error() -> str:

@@ -502,6 +502,27 @@ bp_status bp_check(bp_net* net, void* stream) {
     return fail(BP_ENONFINITE, "the summed squared error of a group was not finite");
 }
 
+bp_status bp_debug_wait_test(bp_net* net, unsigned long long wait_ns, int unreachable) {
+    if (net == nullptr) return fail(BP_EINVAL, "NULL net");
+    if (net->dtype != BP_F32) return fail(BP_EINVAL, "the wait test hook is for float32 nets");
+#ifdef BP_CHECK
+    BP_CUDA(cudaDeviceSynchronize(), "bp_debug_wait_test");
+    net->view.wait_ns = wait_ns;
+    if (unreachable) {
+        // barrier k of the next launch waits for bar[0] + k * grid arrivals
+        unsigned words[2] = {0, 0};
+        BP_CUDA(cudaMemcpy(words, net->bar, sizeof words, cudaMemcpyDeviceToHost), "bp_debug_wait_test");
+        words[0] = words[1] + 0x40000000u;
+        BP_CUDA(cudaMemcpy(net->bar, words, sizeof(unsigned), cudaMemcpyHostToDevice), "bp_debug_wait_test");
+    }
+    return BP_OK;
+#else
+    (void)wait_ns;
+    (void)unreachable;
+    return fail(BP_ESTATE, "bp_debug_wait_test works only in a library built with -DBP_CHECK");
+#endif
+}
+
 bp_status bp_train_epoch_host(bp_net* net, const void* h_X, const void* h_T, int n_patterns,
                               int minibatch, float* h_sse, void* stream) {
     if (net == nullptr || h_X == nullptr || h_T == nullptr) return fail(BP_EINVAL, "NULL argument");

@@ -130,7 +130,7 @@ __device__ __forceinline__ uint32_t smem_u32(const void* p) {
 __device__ __forceinline__ bool count_reached(unsigned v, unsigned target) {
     return (int)(v - target) >= 0;
 }
-__device__ bool grid_barrier(unsigned* bar, unsigned target, int* flags) {
+__device__ bool grid_barrier(unsigned* bar, unsigned target, int* flags, unsigned long long limit_ns) {
     __syncthreads();
     int ok = 1;
     if (threadIdx.x == 0) {
@@ -140,7 +140,7 @@ __device__ bool grid_barrier(unsigned* bar, unsigned target, int* flags) {
         unsigned it = 0;
         while (!count_reached(ld_acquire(bar + 1), target)) {
             ++it;
-            if (it > kWaitIters || ((it & 63u) == 0 && global_ns() - t0 > kWaitNs)) {
+            if (it > kWaitIters || ((it & 63u) == 0 && global_ns() - t0 > limit_ns)) {
                 atomicOr(flags, kFlagTimeout);
                 ok = 0;
                 break;
@@ -148,6 +148,18 @@ __device__ bool grid_barrier(unsigned* bar, unsigned target, int* flags) {
         }
     }
     return __syncthreads_and(ok) != 0;
+}
+
+// Limit of the grid barrier's wait: 2 s, or in the checked build the limit a
+// test set on the net (bp_debug_wait_test), so that a test can make a wait run
+// out in about a millisecond.
+__device__ __forceinline__ unsigned long long wait_limit_ns(const F32View& v) {
+#ifdef BP_CHECK
+    return v.wait_ns != 0 ? v.wait_ns : kWaitNs;
+#else
+    (void)v;
+    return kWaitNs;
+#endif
 }
 
 __device__ __forceinline__ float warp_sum(float x) {
@@ -180,24 +192,39 @@ __device__ __forceinline__ void mbar_init1(uint64_t* bar) {
     __syncthreads();
 }
 
+__device__ __forceinline__ bool mbar_try(uint64_t* bar, unsigned parity) {
+    unsigned done;
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+        "selp.u32 %0, 1, 0, p;\n\t}"
+        : "=r"(done)
+        : "r"(smem_u32(bar)), "r"(parity)
+        : "memory");
+    return done != 0;
+}
+
 // Waits (bounded) for the phase with the given parity of an mbarrier; on a
-// timeout latches kFlagTimeout and returns false.
+// timeout latches kFlagTimeout and returns false.  The copy it waited for may
+// then still be in flight: the caller issues no more copies and drains
+// (mbar_drain) every copy it issued before the CTA may return.
 __device__ __forceinline__ bool mbar_wait(uint64_t* bar, unsigned parity, int* flags) {
-    unsigned done = 0;
     const unsigned long long t0 = global_ns();
     for (unsigned it = 0;; ++it) {
-        asm volatile(
-            "{\n\t.reg .pred p;\n\t"
-            "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
-            "selp.u32 %0, 1, 0, p;\n\t}"
-            : "=r"(done)
-            : "r"(smem_u32(bar)), "r"(parity)
-            : "memory");
-        if (done) return true;
+        if (mbar_try(bar, parity)) return true;
         if ((it & 255u) == 255u && global_ns() - t0 > kWaitNs) {
             atomicOr(flags, kFlagTimeout);
             return false;
         }
+    }
+}
+
+// Second bounded wait for a copy whose first wait ran out, so that its bulk
+// writes land before the CTA exits (shared memory of an exited CTA may belong
+// to the next CTA on that SM).  The error is already latched.
+__device__ __forceinline__ void mbar_drain(uint64_t* bar, unsigned parity) {
+    const unsigned long long t0 = global_ns();
+    while (!mbar_try(bar, parity) && global_ns() - t0 < kWaitNs) {
     }
 }
 
@@ -222,24 +249,43 @@ __device__ void stage_weights_issue(const float* theta, long long P, float* Ws, 
 }
 
 // Bounded wait for a copy started by stage_weights_issue (every thread; the
-// tail written by plain stores needs a CTA barrier after this).
+// tail written by plain stores needs a CTA barrier after this).  Returns false
+// in a thread whose wait ran out; callers make that CTA-uniform with
+// __syncthreads_or and then call stage_weights_drain before returning.
 struct WeightCopy {
     uint64_t* bar;
     unsigned* phase;
     long long P;
 };
-__device__ __forceinline__ void stage_weights_wait(const WeightCopy& w, int* flags) {
+__device__ __forceinline__ bool stage_weights_wait(const WeightCopy& w, int* flags) {
+    bool ok = true;
     if ((w.P & ~3LL) > 0) {
-        mbar_wait(w.bar, *w.phase, flags);
+        ok = mbar_wait(w.bar, *w.phase, flags);
         *w.phase ^= 1u;
     }
+    return ok;
 }
 
-__device__ void stage_weights(const float* theta, long long P, float* Ws, uint64_t* bar,
+// After a weight copy whose wait ran out in some thread: thread 0 waits for
+// that copy again (bounded) so that no bulk write is still landing when the CTA
+// returns.  Every thread calls it.
+__device__ void stage_weights_drain(const WeightCopy& w) {
+    if (threadIdx.x == 0 && (w.P & ~3LL) > 0) mbar_drain(w.bar, *w.phase ^ 1u);
+    __syncthreads();
+}
+
+// Copies the weights into shared memory and waits for them; false (in every
+// thread) if the copy timed out, in which case it has been drained and the
+// caller must return.
+__device__ bool stage_weights(const float* theta, long long P, float* Ws, uint64_t* bar,
                               unsigned& phase, int* flags) {
     stage_weights_issue(theta, P, Ws, bar);
-    stage_weights_wait(WeightCopy{bar, &phase, P}, flags);
-    __syncthreads();
+    const WeightCopy wc{bar, &phase, P};
+    if (__syncthreads_or(!stage_weights_wait(wc, flags))) {
+        stage_weights_drain(wc);
+        return false;
+    }
+    return true;
 }
 
 // ------------------------------------------------------------ pattern phase
@@ -449,12 +495,15 @@ __device__ __forceinline__ void rows_to_scratch(const F32View& v, int l, const f
 //   to_scratch: write the activation and delta rows to scratch (A, D)
 //   rows_issued: the first pass's rows were already issued (load_rows)
 //   whole: this CTA takes all B patterns (diagnostic mode) instead of its share
+//   copy_ok: with wc, set false (in every thread) if the weight copy timed out;
+//       it has then been drained and the phase did nothing, so the caller returns
 template <int PG>
 __device__ float pattern_phase(const F32View& v, const PatLayout& q, const float* Wb,
                                const float* __restrict__ X, const float* __restrict__ T, int B,
                                bool do_fwd, bool do_bwd, float* __restrict__ Y, float* smem,
                                const WeightCopy* wc = nullptr, bool to_scratch = true,
-                               bool rows_issued = false, bool whole = false) {
+                               bool rows_issued = false, bool whole = false,
+                               bool* copy_ok = nullptr) {
     constexpr int TP = kThreads / PG;
     const int L = v.L;
     const int tid = threadIdx.x;
@@ -463,10 +512,15 @@ __device__ float pattern_phase(const F32View& v, const PatLayout& q, const float
     float sse = 0.f;
     const int q_lo = whole ? 0 : (int)((long long)B * blockIdx.x / gridDim.x);
     const int q_hi = whole ? B : (int)((long long)B * (blockIdx.x + 1) / gridDim.x);
+    if (copy_ok != nullptr) *copy_ok = true;
     if (!bounds_ok((size_t)(smem - pattern_smem_base()) + q.total <= dyn_smem_floats() &&
                        ((!to_scratch && do_fwd) || B <= v.cap),
                    v.flags)) {
-        if (wc != nullptr) stage_weights_wait(*wc, v.flags);
+        if (wc != nullptr && __syncthreads_or(!stage_weights_wait(*wc, v.flags))) {
+            stage_weights_drain(*wc);
+            if (copy_ok != nullptr) *copy_ok = false;
+            return 0.f;
+        }
         return block_sum(0.f);
     }
     for (int p0 = q_lo; p0 < q_hi; p0 += PG) {
@@ -482,12 +536,19 @@ __device__ float pattern_phase(const F32View& v, const PatLayout& q, const float
                     dst[c] = (pr < np) ? __ldcg(act_chunk(v, l, p0 + pr, c)) : make_float4(0.f, 0.f, 0.f, 0.f);
             }
         }
+        bool w_ok = true;
+        const WeightCopy* waited = wc;
         if (wc != nullptr) {
-            stage_weights_wait(*wc, v.flags);
+            w_ok = stage_weights_wait(*wc, v.flags);
             wc = nullptr;
         }
         cp_async_wait<0>();
-        __syncthreads();
+        if (__syncthreads_or(!w_ok)) {
+            // the weight copy did not arrive in time: let it land, do nothing more
+            stage_weights_drain(*waited);
+            if (copy_ok != nullptr) *copy_ok = false;
+            return 0.f;
+        }
         if (do_fwd) {
             for (int l = 1; l <= L; ++l) {
                 forward_layer<PG>(Wb + v.woff[l], v.kp[l], v.n[l], smem + q.sa[l - 1], smem + q.sa[l],
@@ -530,7 +591,11 @@ __device__ float pattern_phase(const F32View& v, const PatLayout& q, const float
         }
         __syncthreads();
     }
-    if (wc != nullptr) stage_weights_wait(*wc, v.flags);   // no patterns here
+    if (wc != nullptr && __syncthreads_or(!stage_weights_wait(*wc, v.flags))) {   // no patterns here
+        stage_weights_drain(*wc);
+        if (copy_ok != nullptr) *copy_ok = false;
+        return 0.f;
+    }
     // the weight phase reads the activation and delta rows through TMA
     asm volatile("fence.proxy.async.global;" ::: "memory");
     return block_sum(sse);
@@ -598,7 +663,11 @@ __device__ __forceinline__ void issue_chunk(const F32View& v, ChunkPipe& pipe, f
 // meet by a butterfly inside the warp.  The blocks' row chunks are stored
 // permuted by pattern (see F32View), which keeps the lanes' reads of 32
 // consecutive rows free of bank conflicts.
-__device__ void weight_phase(const F32View& v, int B, bool fused, bool fold_g, float* smem,
+//
+// Returns false (in every thread) if a chunk copy did not arrive in time: no
+// more copies are then issued, every copy already issued has been drained, no
+// weight was written for the tile, and the caller must return.
+__device__ bool weight_phase(const F32View& v, int B, bool fused, bool fold_g, float* smem,
                              ChunkPipe& pipe) {
     const int tid = threadIdx.x;
     const int lane = tid & 31, warp = tid >> 5;
@@ -610,7 +679,7 @@ __device__ void weight_phase(const F32View& v, int B, bool fused, bool fold_g, f
     if (!bounds_ok((size_t)(wbuf - pattern_smem_base()) + kNBuf * kChunkFloats <= dyn_smem_floats() &&
                        B <= v.cap,
                    v.flags))
-        return;
+        return true;
     for (int t = blockIdx.x; t < ntiles; t += gridDim.x) {
         int l = 1;
         while (t >= v.tile0[l + 1]) ++l;
@@ -619,7 +688,7 @@ __device__ void weight_phase(const F32View& v, int B, bool fused, bool fold_g, f
         const int n_in = v.n[l - 1], n_out = v.n[l];
         const int u0 = tb * kTU, j0 = cb * kTJ;
         // the tile's blocks exist in the scratch layout
-        if (!bounds_ok(tb < v.dtb[l] && cb < v.acb[l - 1], v.flags)) return;
+        if (!bounds_ok(tb < v.dtb[l] && cb < v.acb[l - 1], v.flags)) return true;
         // this lane's output (lanes 0..15 of each warp) and its current weight
         // state, loaded now so that their latency hides behind the chunks
         const int uu = u0 + uq * 4 + ((lane & 15) >> 2), ii = j0 + cq * 4 + (lane & 3);
@@ -644,7 +713,7 @@ __device__ void weight_phase(const F32View& v, int B, bool fused, bool fold_g, f
         }
         for (int c = 0; c < nchunks; ++c) {
             const int b = c % kNBuf;
-            mbar_wait(pipe.bar + b, (pipe.parity >> b) & 1u, v.flags);
+            const bool got = mbar_wait(pipe.bar + b, (pipe.parity >> b) & 1u, v.flags);
             pipe.parity ^= 1u << b;
             float* As = wbuf + b * kChunkFloats;
             float* Ds = As + kPC * kTJ;
@@ -667,7 +736,20 @@ __device__ void weight_phase(const F32View& v, int B, bool fused, bool fold_g, f
 #pragma unroll
                     for (int q = 0; q < 4; ++q) acc[u * 4 + q] = fmaf(dv[u], av[q], acc[u * 4 + q]);
             }
-            __syncthreads();
+            if (__syncthreads_or(!got)) {
+                // a chunk did not arrive in time: issue nothing more and let
+                // every copy already issued land (chunks c + 1 .. c + kNBuf - 1,
+                // and chunk c if thread 0 did not see it complete)
+                if (tid == 0) {
+                    if (!got) mbar_drain(pipe.bar + b, ((pipe.parity >> b) & 1u) ^ 1u);
+                    for (int k = c + 1; k < nchunks && k < c + kNBuf; ++k) {
+                        const int bk = k % kNBuf;
+                        mbar_drain(pipe.bar + bk, (pipe.parity >> bk) & 1u);
+                    }
+                }
+                __syncthreads();
+                return false;
+            }
             if (tid == 0 && c + kNBuf < nchunks) {
                 asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
                 issue_chunk(v, pipe, wbuf, l, tb, cb, c + kNBuf, min(kPC, B - (c + kNBuf) * kPC));
@@ -697,6 +779,7 @@ __device__ void weight_phase(const F32View& v, int B, bool fused, bool fold_g, f
             asm volatile("fence.proxy.async.global;" ::: "memory");
         }
     }
+    return true;
 }
 
 // Initialises the weight-phase mbarriers (static shared memory) of a launch.
@@ -738,7 +821,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (WS) {
         mbar_init1(&s_bar);
         if (!bounds_ok((unsigned)v.wsm <= dyn_smem_floats(), v.flags)) return;
-        stage_weights(v.theta, v.P, smem, &s_bar, phase, v.flags);
+        if (!stage_weights(v.theta, v.P, smem, &s_bar, phase, v.flags)) return;
         pattern_phase<PG>(v, q, smem, X, nullptr, B, true, false, Y, pattern_base<true>(v, smem));
     } else {
         pattern_phase<PG>(v, q, v.theta, X, nullptr, B, true, false, Y, pattern_base<false>(v, smem));
@@ -755,7 +838,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (WS) {
         mbar_init1(&s_bar);
         if (!bounds_ok((unsigned)v.wsm <= dyn_smem_floats(), v.flags)) return;
-        stage_weights(v.theta, v.P, smem, &s_bar, phase, v.flags);
+        if (!stage_weights(v.theta, v.P, smem, &s_bar, phase, v.flags)) return;
         e = pattern_phase<PG>(v, q, smem, nullptr, T, B, false, true, nullptr, pattern_base<true>(v, smem));
     } else {
         e = pattern_phase<PG>(v, q, v.theta, nullptr, T, B, false, true, nullptr, pattern_base<false>(v, smem));
@@ -778,7 +861,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (WS && !bounds_ok((unsigned)v.wsm <= dyn_smem_floats(), v.flags)) return;
     float e;
     if (WS) {
-        stage_weights(v.theta, v.P, smem, &s_bar, phase, v.flags);
+        if (!stage_weights(v.theta, v.P, smem, &s_bar, phase, v.flags)) return;
         e = pattern_phase<PG>(v, q, smem, X, T, B, true, true, nullptr, pattern_base<true>(v, smem),
                               nullptr, false, false, true);
     } else {
@@ -800,7 +883,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     ChunkPipe pipe;
     pipe_init(pipe, s_cbar);
     reduce_sse(v, nparts, sse_out);
-    weight_phase(v, B, false, false, smem, pipe);
+    weight_phase(v, B, false, false, smem, pipe);   // on a timeout it has drained its copies
 }
 
 __global__ void __launch_bounds__(256) k_update(const __grid_constant__ F32View v, long long n) {
@@ -843,16 +926,19 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (WS) {
             stage_weights_issue(v.theta, v.P, smem, &s_bar);
             const WeightCopy wc{&s_bar, &phase, v.P};
-            e = pattern_phase<PG>(v, q, smem, Xs, Ts, B, true, true, nullptr, pat, &wc);
+            bool copy_ok = true;
+            e = pattern_phase<PG>(v, q, smem, Xs, Ts, B, true, true, nullptr, pat, &wc, true, false,
+                                  false, &copy_ok);
+            if (!copy_ok) return;   // the copy was drained; the error is latched
         } else {
             e = pattern_phase<PG>(v, q, v.theta, Xs, Ts, B, true, true, nullptr, pat);
         }
         if (threadIdx.x == 0) v.sse_part[blockIdx.x] = e;
-        if (!grid_barrier(v.bar, target += gridDim.x, v.flags)) return;
+        if (!grid_barrier(v.bar, target += gridDim.x, v.flags, wait_limit_ns(v))) return;
         reduce_sse(v, gridDim.x, sse_out != nullptr ? sse_out + s : nullptr);
-        weight_phase(v, B, true, fold_g != 0 && s == 0, smem, pipe);
+        if (!weight_phase(v, B, true, fold_g != 0 && s == 0, smem, pipe)) return;
         if (s + 1 < n_steps) {
-            if (!grid_barrier(v.bar, target += gridDim.x, v.flags)) return;
+            if (!grid_barrier(v.bar, target += gridDim.x, v.flags, wait_limit_ns(v))) return;
         }
     }
     // every CTA has passed a barrier, so every CTA has read bar[0]: publish the
@@ -905,7 +991,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         vel[m] = live ? reinterpret_cast<const float4*>(v.V + v.woff[l] + (long long)j * v.kp[l])[c]
                       : make_float4(0.f, 0.f, 0.f, 0.f);
     }
-    stage_weights(v.theta, v.P, smem, &s_bar, phase, v.flags);
+    if (!stage_weights(v.theta, v.P, smem, &s_bar, phase, v.flags)) return;
     const float a_lr = v.lr * v.grad_scale, mom = v.momentum, guard = v.guard;
     if (n_steps > 0)
         load_rows<PG>(v, q, X, T, 0, (int)min((long long)minibatch, (long long)n_patterns), pat[0]);

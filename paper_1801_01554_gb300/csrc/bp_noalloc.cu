@@ -86,6 +86,18 @@ extern "C" bp_status bp_train_epoch_noalloc(const int* layer_sizes, int n_layers
         set_error_message("bp_train_epoch_noalloc: n_patterns and minibatch must be >= 1");
         return BP_EINVAL;
     }
+    // the kernels read and write these as float32 words (4-byte cp.async for
+    // the pattern rows): refuse a misaligned pointer before any CUDA call
+    {
+        const void* p[6] = {d_theta, d_V, d_X, d_T, d_sse, d_status};
+        const char* what[6] = {"d_theta", "d_V", "d_X", "d_T", "d_sse", "d_status"};
+        for (int k = 0; k < 6; ++k)
+            if (((uintptr_t)p[k] & 3u) != 0) {
+                snprintf(msg, sizeof msg, "bp_train_epoch_noalloc: %s must be 4-byte aligned", what[k]);
+                set_error_message(msg);
+                return BP_EINVAL;
+            }
+    }
     const int L = n_layers - 1;
     if (f32_max_pg(layer_sizes, L) < 1) {
         set_error_message("bp_train_epoch_noalloc: one pattern's activations do not fit in shared memory");

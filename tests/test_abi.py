@@ -74,3 +74,22 @@ def test_null_handles_are_rejected(lib):
     assert lib.bp_set_guard(None, 1.0) == bp.BP_EINVAL
     assert lib.bp_get_faults(None, None, 0) == bp.BP_EINVAL
     lib.bp_destroy(None)   # NULL-safe
+
+
+@pytest.mark.parametrize("bad", ["d_theta", "d_V", "d_X", "d_T", "d_sse", "d_status"])
+def test_noalloc_rejects_misaligned_pointers_before_any_cuda_call(lib, bad):
+    """The allocation-free entry point reads its buffers as float32 words: a
+    pointer off a 4-byte boundary is refused with BP_EINVAL before the call
+    touches the device (this runs without a GPU, so any CUDA call would fail
+    with BP_ECUDA instead).  The addresses are never dereferenced."""
+    sizes = (203, 120, 26)
+    arr = (ctypes.c_int * 3)(*sizes)
+    ptrs = {k: 0x10000 * (i + 1) for i, k in enumerate(["d_theta", "d_V", "d_X", "d_T", "d_sse",
+                                                        "d_status"])}
+    ptrs[bad] += 2
+    st = lib.bp_train_epoch_noalloc(arr, 3, 0.05, 0.9, 1.0, ptrs["d_theta"], ptrs["d_V"],
+                                    ptrs["d_X"], ptrs["d_T"], 512, 512, ptrs["d_sse"],
+                                    ptrs["d_status"], None)
+    assert st == bp.BP_EINVAL
+    msg = lib.bp_last_error().decode()
+    assert bad in msg and "aligned" in msg
