@@ -1,26 +1,31 @@
 """bfloat16 tensor-core path against the float64 oracle, through the C ABI.
 
-Tolerance (bf16 tensor-core path): normwise relative error <= 2e-2 on outputs
-and on weights after 10 updates; the pooled change is held to the same 2e-2
-(inputs, weight copies, activations and deltas are each rounded to bfloat16,
-unit roundoff 2^-9, and the products accumulate in fp32).
+Tolerance (bf16 tensor-core path): normwise relative error <= 2e-2 on outputs,
+on the error sums, on the pooled change of a step and, per layer, on the weights
+and on the weight change W10 - W0 after 10 updates (inputs, weight copies,
+activations and deltas are each rounded to bfloat16, unit roundoff 2^-9, and
+the products accumulate in fp32).  Errors are taken per layer, separately for
+W_l and b_l (tests/parity.py).
+
+The 10-update runs at the 4096-wide layers use the mean (grad_scale = 1/B):
+with the pooled sum, the first update of a net that wide drives its units into
+saturation, and the float64 oracle's own 10-update weight change then moves by
+more than 100% under a perturbation of the size of one bf16 rounding (pinned on
+the CPU by tests/test_oracle.py), so no rounded path can be held to it there.
+The sum-mode step at those widths is held to the bar on its first update, at
+B = 1024 and at the full batch.
 """
 import numpy as np
 import pytest
 
 from oracle import bp_oracle as O
 from paper_1801_01554_gb300 import bp, synth
+from parity import assert_layers, normwise
 
 torch = pytest.importorskip("torch")
 pytestmark = pytest.mark.gpu
 
 TOL = 2e-2
-
-
-def normwise(x, y):
-    x = np.asarray(x, dtype=np.float64)
-    y = np.asarray(y, dtype=np.float64)
-    return float(np.max(np.abs(x - y)) / max(np.max(np.abs(y)), 1e-30))
 
 
 def dev_bf16(a):
@@ -39,13 +44,16 @@ def problem(sizes, B, seed=0, p_one=0.3):
     return X, T, theta
 
 
-SHAPES = [((64, 128, 32), 200), ((128, 256, 64), 300), ((8, 16, 8), 8), ((200, 136, 72, 24), 1000),
-          ((256, 512, 256), 128), ((1024, 2048, 2048, 512), 1024)]
+SHAPES = [((64, 128, 32), 200, 0.3), ((128, 256, 64), 300, 0.3), ((8, 16, 8), 8, 0.3),
+          ((200, 136, 72, 24), 1000, 0.3), ((256, 512, 256), 128, 0.3),
+          ((1024, 2048, 2048, 512), 1024, 0.1), ((4096,) * 5, 1024, 0.5)]
 
 
-@pytest.mark.parametrize("sizes,B", SHAPES)
-def test_forward_backward_match_oracle(sizes, B):
-    X, T, theta = problem(sizes, B, seed=B)
+@pytest.mark.parametrize("sizes,B,p_one", SHAPES)
+def test_forward_backward_update_match_oracle(sizes, B, p_one):
+    """One step in sum mode: outputs, error sum, the pooled change of every
+    layer, and the update it makes (W1 - W0 and V1 per layer)."""
+    X, T, theta = problem(sizes, B, seed=B, p_one=p_one)
     st = O.State(sizes, theta, lr=0.01, momentum=0.9)
     As, Ds, G_ref, e_ref = O.step_quantities(st, X, T)
     Xd, Td = dev_bf16(X), dev_bf16(T)
@@ -57,26 +65,42 @@ def test_forward_backward_match_oracle(sizes, B):
         net.backward(Td, B, sse)
         net.check()
         G = net.get_grads()
+        net.update()
+        net.check()
+        W1, V1 = net.get_weights(), net.get_velocity()
     y = Yd.float().cpu().numpy()
     assert normwise(y, As[-1]) <= TOL
     assert abs(sse.item() - e_ref) <= TOL * e_ref
-    offs, _ = synth.param_layout(sizes)
-    for l, (w_off, b_off) in enumerate(offs, start=1):
-        n_w = sizes[l] * sizes[l - 1]
-        err_w = normwise(G[w_off:w_off + n_w], G_ref[w_off:w_off + n_w])
-        err_b = normwise(G[b_off:b_off + sizes[l]], G_ref[b_off:b_off + sizes[l]])
-        assert err_w <= TOL, (l, err_w)
-        assert err_b <= TOL, (l, err_b)
+    assert_layers(sizes, G, G_ref, TOL, None, "G")
+    st.G = G_ref
+    O.apply_update(st)
+    assert_layers(sizes, W1 - theta, st.theta - theta, TOL, None, "W1-W0")
+    assert_layers(sizes, V1, st.V, TOL, None, "V1")
 
 
-@pytest.mark.parametrize("sizes,B", [((64, 128, 32), 256), ((200, 136, 72, 24), 520),
-                                     ((1024, 2048, 2048, 512), 1024)])
-def test_ten_updates_match_oracle(sizes, B):
-    X, T, theta = problem(sizes, B, seed=5, p_one=0.1)
+TEN = [((64, 128, 32), 256, 0.1, "sum"), ((200, 136, 72, 24), 520, 0.1, "sum"),
+       ((1024, 2048, 2048, 512), 1024, 0.1, "sum"), ((1024, 2048, 2048, 512), 1024, 0.1, "mean"),
+       ((4096,) * 5, 1024, 0.5, "mean")]
+
+
+@pytest.mark.parametrize("sizes,B,p_one,mode", TEN)
+def test_ten_updates_match_oracle(sizes, B, p_one, mode):
+    """Ten updates on one group: the pooled change of the first step per layer,
+    the weights and the weight change W10 - W0 per layer, and every update's
+    error sum."""
+    X, T, theta = problem(sizes, B, seed=5, p_one=p_one)
     lr, m = 0.01, 0.9
-    st = O.State(sizes, theta, lr=lr, momentum=m)
+    gs = 1.0 if mode == "sum" else 1.0 / B
+    st = O.State(sizes, theta, lr=lr, momentum=m, grad_scale=gs)
+    G_ref = O.step_quantities(st, X, T)[2]
     Xd, Td = dev_bf16(X), dev_bf16(T)
-    with bp.Net(sizes, lr, m, bp.BP_BF16, max_batch=B) as net:
+    with bp.Net(sizes, lr, m, bp.BP_BF16, max_batch=B, grad_scale=gs) as net:
+        net.set_weights(theta)
+        net.forward(Xd, B)
+        net.backward(Td, B)
+        net.check()
+        G1 = net.get_grads()
+    with bp.Net(sizes, lr, m, bp.BP_BF16, max_batch=B, grad_scale=gs) as net:
         net.set_weights(theta)
         sse = torch.zeros(10, device="cuda")
         for k in range(10):
@@ -84,9 +108,10 @@ def test_ten_updates_match_oracle(sizes, B):
         net.check()
         th = net.get_weights()
     e_ref = [O.train_batch(st, X, T) for _ in range(10)]
-    print("W:", normwise(th, st.theta), "W10-W0:", normwise(th - theta, st.theta - theta))
-    assert normwise(th, st.theta) <= TOL
-    assert normwise(th - theta, st.theta - theta) <= 5 * TOL
+    assert_layers(sizes, G1, G_ref, TOL, None, "G1")
+    errs = assert_layers(sizes, th - theta, st.theta - theta, TOL, None, "W10-W0")
+    print("W10-W0 per part:", {k: f"{v:.2e}" for k, v in errs.items()})
+    assert_layers(sizes, th, st.theta, TOL, None, "W10")
     np.testing.assert_allclose(sse.cpu().numpy(), e_ref, rtol=TOL)
 
 
@@ -107,7 +132,7 @@ def test_separate_calls_equal_train_batch():
                     net.update()
             net.check()
             out.append(net.get_weights())
-    assert normwise(out[1] - theta, out[0] - theta) <= 1e-3
+    assert_layers(sizes, out[1] - theta, out[0] - theta, 1e-3, None, "separate vs fused")
 
 
 def test_epoch_of_minibatches_matches_oracle():
@@ -122,7 +147,7 @@ def test_epoch_of_minibatches_matches_oracle():
         net.check()
         th = net.get_weights()
     np.testing.assert_allclose(sse.cpu().numpy(), e_ref, rtol=TOL)
-    assert normwise(th - theta, st.theta - theta) <= 5 * TOL
+    assert_layers(sizes, th - theta, st.theta - theta, TOL, None, "epoch W-W0")
 
 
 def test_pooled_change_adds_over_groups():
@@ -167,10 +192,12 @@ def test_runs_are_bitwise_reproducible():
 
 @pytest.mark.slow
 @pytest.mark.parametrize("name", ["wide3", "wide4096"])
-def test_full_size_workload_sampled(name):
-    """Full batch size, launched as the training step is: outputs of sampled
-    patterns against the oracle's forward pass of those patterns; the error sum
-    of the step against the sum over the path's own outputs."""
+def test_full_size_step_matches_oracle(name):
+    """The benchmark's workload at its full batch, launched as bench.py times
+    it (bp_train_batch on the whole group, sum mode): outputs of sampled
+    patterns against the oracle's forward pass of those patterns, then one
+    training step -- its error sum and the weight change of every layer --
+    against the oracle's full step (6.6 TFLOP in float64 for 4096^5)."""
     sizes, X, T, theta = synth.make_workload(name)
     w = synth.WORKLOADS[name]
     B = w["minibatch"]
@@ -185,15 +212,17 @@ def test_full_size_workload_sampled(name):
         net.check()
         y = Yd.float().cpu().numpy()
         assert normwise(y[rows], y_ref) <= TOL
-        sse = torch.zeros(2, device="cuda")
-        net.train_batch(Xd, Td, B, sse[0:1])
-        net.train_batch(Xd, Td, B, sse[1:2])
+        sse = torch.zeros(1, device="cuda")
+        net.train_batch(Xd, Td, B, sse)
         net.check()
         th = net.get_weights()
-    assert np.all(np.isfinite(th))
-    assert np.any(th != theta.astype(np.float32))
-    e_own = float(np.sum((T - y) ** 2))
-    assert abs(sse[0].item() - e_own) <= 1e-3 * e_own
+    del Xd, Td, Yd
+    torch.cuda.empty_cache()
+    st = O.State(sizes, theta, lr=w["lr"], momentum=w["momentum"])
+    e_ref = O.train_batch(st, X, T)
+    assert abs(sse.item() - e_ref) <= TOL * e_ref
+    errs = assert_layers(sizes, th - theta, st.theta - theta, TOL, None, "W1-W0")
+    print(name, "W1-W0 per part:", {k: f"{v:.2e}" for k, v in errs.items()})
 
 
 def test_fault_guard_zeroes_and_counts_on_the_bf16_update():
@@ -217,7 +246,7 @@ def test_fault_guard_zeroes_and_counts_on_the_bf16_update():
         assert net.get_faults() == 0
         st = O.State(sizes, theta, lr=0.05, momentum=0.9)
         O.train_batch(st, X, T)
-        assert normwise(net.get_weights() - theta, st.theta - theta) <= TOL
+        assert_layers(sizes, net.get_weights() - theta, st.theta - theta, TOL, None, "W-W0")
 
 
 def test_deepest_net_the_boundary_allows():
@@ -238,7 +267,7 @@ def test_deepest_net_the_boundary_allows():
         net.train_batch(Xd, Td, B)
         net.check()
         assert normwise(Y.float().cpu().numpy(), Y_ref) <= TOL
-        assert normwise(net.get_weights() - theta, st.theta - theta) <= TOL
+        assert_layers(sizes, net.get_weights() - theta, st.theta - theta, TOL, None, "W1-W0")
 
 
 def test_misaligned_pattern_buffers_are_rejected_before_any_launch():
@@ -263,4 +292,4 @@ def test_misaligned_pattern_buffers_are_rejected_before_any_launch():
         net.check()
         st = O.State(sizes, theta, lr=0.05, momentum=0.9)
         O.train_batch(st, X, T)
-        assert normwise(net.get_weights() - theta, st.theta - theta) <= TOL
+        assert_layers(sizes, net.get_weights() - theta, st.theta - theta, TOL, None, "W1-W0")

@@ -332,3 +332,55 @@ def test_guarded_update_skips_only_the_zeroed_weights():
     assert st.faults == int(big.sum()) > 0
     np.testing.assert_array_equal(st.theta[big], theta[big])
     np.testing.assert_allclose(st.theta[~big], theta[~big] + 0.5 * G[~big], rtol=0, atol=1e-15)
+
+
+def _trajectory_sensitivity(width, B, grad_scale):
+    """Relative change, per part, of the oracle's 10-update weight change on a
+    width^5 net (bf16 inputs, Bernoulli(0.5) targets, N(0, 1/fan_in) weights,
+    lr 0.01, momentum 0.9) when the initial weights move by one bf16 rounding."""
+    import sys
+    sys.path.insert(0, os.path.dirname(__file__))
+    from parity import layer_errors
+    sizes = (width,) * 5
+    X, T = synth.gaussian_patterns(B, width, width, 0.5, seed=5)
+    X = synth.round_to(X, "bf16")
+    theta = synth.round_to(synth.init_normal_fanin(sizes, 5), "f32")
+    thp = theta * (1 + np.random.default_rng(7).uniform(-2.0 ** -9, 2.0 ** -9, theta.size))
+    dws = []
+    for th in (theta, thp):
+        st = O.State(sizes, th, lr=0.01, momentum=0.9, grad_scale=grad_scale)
+        for _ in range(10):
+            O.train_batch(st, X, T)
+        dws.append(st.theta - th)
+    return layer_errors(sizes, dws[1], dws[0])
+
+
+def test_wide_sum_mode_trajectory_is_ill_conditioned_and_mean_mode_is_not():
+    """The reading behind the bf16 10-update parity runs: with the pooled sum,
+    the first update of a wide net drives its units into saturation, and the
+    exact 10-update weight change of the output layer then moves by more than
+    50% when the initial weights move by one bf16 rounding (2^-9), so a
+    bf16 path cannot be held to it; with the mean the same perturbation moves
+    every layer's change by under 1%."""
+    s = _trajectory_sensitivity(512, 1024, 1.0)
+    assert s["W4"] > 0.5
+    m = _trajectory_sensitivity(512, 1024, 1.0 / 1024)
+    assert max(m.values()) < 1e-2
+
+
+def test_case_parallel_driver_equals_the_serial_oracle():
+    """Section 4.1's case parallelism: the changes of the workers' shares of
+    each group, summed, give the serial oracle's update (up to the order of
+    the float64 sums), ragged last group included."""
+    from oracle.case_parallel import CaseParallel
+    sizes, n, mb = (203, 30, 26), 700, 128
+    X, T = synth.nettalk_patterns(n, seed=3)
+    theta = synth.init_uniform(sizes, -0.3, 0.3, 3)
+    a = O.State(sizes, theta, lr=0.05, momentum=0.9)
+    e_ref = O.train_epoch(a, X, T, mb)
+    b = O.State(sizes, theta, lr=0.05, momentum=0.9)
+    with CaseParallel(sizes, X, T, workers=3) as cp:
+        e = cp.train_epoch(b, n, mb)
+    np.testing.assert_allclose(e, e_ref, rtol=1e-12)
+    np.testing.assert_allclose(b.theta, a.theta, rtol=0, atol=1e-12)
+    np.testing.assert_allclose(b.V, a.V, rtol=0, atol=1e-12)

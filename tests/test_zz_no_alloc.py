@@ -61,3 +61,43 @@ def test_noalloc_rejects_sizes_beyond_its_scratch():
         bp.bp_train_epoch_noalloc(sizes, 0.1, 0.9, 1.0, th, th.clone(), X, T, 16, 100000)
     assert e.value.status == bp.BP_EINVAL
     assert "scratch" in bp.bp_last_error()
+
+
+def test_noalloc_smaller_call_after_a_larger_one():
+    """The static scratch keeps the previous call's activations, deltas and
+    padded weights.  A call on a larger net and minibatch, then one on a
+    smaller, deeper net: the second must give the same bits as
+    bp_train_epoch on a fresh net (same kernel, same plan), so nothing stale
+    from the first call reaches it."""
+    big, n1, mb1 = (203, 120, 26), 4096, 2048
+    X1, T1 = synth.nettalk_patterns(n1, seed=31)
+    th1 = torch.tensor(synth.round_to(synth.init_uniform(big, -0.3, 0.3, 31), "f32"),
+                       dtype=torch.float32, device="cuda")
+    bp.bp_train_epoch_noalloc(big, 0.05, 0.9, 1.0, th1, torch.zeros_like(th1),
+                              torch.tensor(X1, dtype=torch.float32, device="cuda"),
+                              torch.tensor(T1, dtype=torch.float32, device="cuda"), n1, mb1)
+    torch.cuda.synchronize()
+
+    small, n, mb = (64, 33, 17, 9), 300, 100
+    X, T = synth.gaussian_patterns(n, small[0], small[-1], 0.3, seed=32)
+    X = synth.round_to(X, "f32")
+    theta = synth.round_to(synth.init_uniform(small, -0.5, 0.5, 32), "f32")
+    Xd = torch.tensor(X, dtype=torch.float32, device="cuda")
+    Td = torch.tensor(T, dtype=torch.float32, device="cuda")
+    steps = -(-n // mb)
+    with bp.Net(small, 0.05, 0.9, bp.BP_F32, max_batch=mb) as net:
+        net.set_weights(theta)
+        sse_ref = torch.zeros(steps, device="cuda")
+        net.train_epoch(Xd, Td, n, mb, sse_ref)
+        net.check()
+        w_ref, v_ref = net.get_weights(), net.get_velocity()
+    th = torch.tensor(theta, dtype=torch.float32, device="cuda")
+    V = torch.zeros_like(th)
+    sse = torch.zeros(steps, device="cuda")
+    status = torch.full((1,), -1, dtype=torch.int32, device="cuda")
+    bp.bp_train_epoch_noalloc(small, 0.05, 0.9, 1.0, th, V, Xd, Td, n, mb, sse, status)
+    torch.cuda.synchronize()
+    assert int(status.item()) == 0
+    np.testing.assert_array_equal(th.cpu().numpy(), w_ref)
+    np.testing.assert_array_equal(V.cpu().numpy(), v_ref)
+    np.testing.assert_array_equal(sse.cpu().numpy(), sse_ref.cpu().numpy())
