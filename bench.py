@@ -1,9 +1,14 @@
 """Benchmark: back-propagation training throughput in connections per second.
 
-Workload (default): 203-120-26 sigmoid MLP (NETtalk-shaped), float32,
-65,536 synthetic patterns, minibatch 512, lr 0.05, momentum 0.9.  One bench
-step = one epoch = 128 training updates of 512 patterns, run as one persistent
-launch of the library's training kernel through the C ABI.
+Headline workload: 203-120-26 sigmoid MLP (NETtalk-shaped), float32, 65,536
+synthetic patterns, minibatch 512, lr 0.05, momentum 0.9, 5 epochs.  One bench
+step = the workload's 5 epochs = 640 training updates, run as 5 persistent
+launches (one per epoch) of the library's training kernel through the C ABI.
+The same JSON line carries a `configs` object with the other workloads:
+203-60-26 (one step = its 10 full-batch epochs), the group-size sweep on
+203-120-26, and the bf16 nets 1024-2048-2048-512 and 4096^5 (one step = one
+update of the full batch), each with its roofline, CPU baseline and end-to-end
+figure through the host-buffer entry point.
 
 Connections per second follow the paper's definition (Section 7.1): the number
 of connections, bias connections included, times the patterns presented,
@@ -72,7 +77,7 @@ class ClockSampler:
         try:
             self.proc = subprocess.Popen(
                 ["nvidia-smi", "-i", str(self.gpu), f"--query-gpu={self.QUERY}",
-                 "--format=csv,noheader,nounits", "-lms", "100"],
+                 "--format=csv,noheader,nounits", "-lms", "20"],
                 stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
         except (OSError, FileNotFoundError):
             self.proc = None
@@ -149,57 +154,120 @@ def allreduce_max(x, world, device):
 
 
 # ------------------------------------------------------------------ oracle timing
-def _oracle_child(patterns_cap, budget_s, steps=1, warmup=0, min_s=0.0, max_epochs=1,
-                  workload=WORKLOAD):
-    """Runs in a fresh interpreter with one BLAS thread: times the oracle on the
-    leading `patterns_cap` patterns of the workload (one update per minibatch),
-    `warmup` untimed then `steps` timed times, each bounded by `budget_s`."""
+THREAD_VARS = ("OMP_NUM_THREADS", "OPENBLAS_NUM_THREADS", "MKL_NUM_THREADS")
+
+
+def _cpu_child(spec):
+    """Runs in a fresh interpreter: times the CPU oracle on a bounded sample of a
+    workload and returns {"patterns", "seconds", "cores"}.
+
+    spec["mode"]: "serial" (the oracle as it stands, one BLAS thread),
+    "case_parallel" (Section 4.1's scheme: oracle/case_parallel.py with
+    spec["workers"] processes of one thread each) or "blas" (the oracle with
+    numpy's BLAS on every host core).  Groups of spec["minibatch"] patterns of
+    the workload's first spec["patterns"] are taken in index order, epoch after
+    epoch, until at least spec["min_s"] seconds have passed at an epoch's end
+    (or spec["max_s"] at a group's end); spec["groups"] > 0 times exactly that
+    many groups instead.  The all-core modes first run one untimed group (worker
+    start-up, BLAS thread pools)."""
     from oracle import bp_oracle as O
     from paper_1801_01554_gb300 import synth
-    w = synth.WORKLOADS[workload]
-    sizes, X, T, theta = synth.make_workload(workload, patterns=patterns_cap)
+    w = synth.WORKLOADS[spec["workload"]]
+    sizes, X, T, theta = synth.make_workload(spec["workload"], patterns=spec["patterns"])
+    mb = spec["minibatch"]
+    n = len(X)
     st = O.State(sizes, theta, lr=w["lr"], momentum=w["momentum"])
-    mb = w["minibatch"]
-    out = []
-    for k in range(warmup + steps):
-        done = 0
+    cp = None
+    if spec["mode"] == "case_parallel":
+        from oracle.case_parallel import CaseParallel
+        cp = CaseParallel(sizes, X, T, workers=spec["workers"])
+        step = lambda p0, nb: cp.train_batch(st, p0, nb)  # noqa: E731
+        cores = spec["workers"]
+    else:
+        step = lambda p0, nb: O.train_batch(st, X[p0:p0 + nb], T[p0:p0 + nb])  # noqa: E731
+        cores = 1 if spec["mode"] == "serial" else (os.cpu_count() or 1)
+    try:
+        if spec["mode"] != "serial":
+            step(0, min(mb, n))                  # warm-up: worker start, BLAS threads
+        done, g = 0, 0
+        groups_per_epoch = -(-n // mb)
         t0 = time.perf_counter()
-        # cycle through the patterns in index order (epoch after epoch) until at
-        # least min_s seconds have passed, at most max_epochs epochs
         while True:
-            p0 = done % len(X)
-            O.train_batch(st, X[p0:p0 + mb], T[p0:p0 + mb])
-            done += min(mb, len(X) - p0)
+            p0 = (g % groups_per_epoch) * mb
+            nb = min(mb, n - p0)
+            step(p0, nb)
+            done += nb
+            g += 1
             el = time.perf_counter() - t0
-            if el > budget_s or done >= max_epochs * len(X) or (el >= min_s and done % len(X) == 0):
+            if spec.get("groups", 0) > 0:
+                if g >= spec["groups"]:
+                    break
+            elif el >= spec["max_s"] or (el >= spec["min_s"] and p0 + nb == n):
                 break
-        if k >= warmup:
-            out.append({"patterns": done, "seconds": time.perf_counter() - t0})
-    return out
+        return {"patterns": done, "seconds": time.perf_counter() - t0, "cores": cores}
+    finally:
+        if cp is not None:
+            cp.close()
 
 
-def time_oracle(patterns_cap, budget_s, steps=1, warmup=0, min_s=0.0, max_epochs=1,
-                workload=WORKLOAD):
+def time_cpu(spec):
     env = dict(os.environ)
-    for k in ("OMP_NUM_THREADS", "OPENBLAS_NUM_THREADS", "MKL_NUM_THREADS"):
-        env[k] = "1"
+    if spec["mode"] == "blas":
+        for k in THREAD_VARS:
+            env.pop(k, None)
+    else:
+        env.update({k: "1" for k in THREAD_VARS})
     code = ("import json,sys; sys.path.insert(0, %r); import bench; "
-            "print(json.dumps(bench._oracle_child(%d, %f, %d, %d, %f, %d, %r)))"
-            % (ROOT, patterns_cap, budget_s, steps, warmup, min_s, max_epochs, workload))
-    r = subprocess.run([sys.executable, "-c", code], env=env, capture_output=True, text=True,
-                       cwd=ROOT, timeout=1800)
+            "print(json.dumps(bench._cpu_child(json.loads(sys.argv[1]))))" % ROOT)
+    r = subprocess.run([sys.executable, "-c", code, json.dumps(spec)], env=env, capture_output=True,
+                       text=True, cwd=ROOT, timeout=1800)
     if r.returncode != 0:
         raise RuntimeError("oracle timing failed: " + r.stderr[-2000:])
     return json.loads(r.stdout.strip().splitlines()[-1])
 
 
-# DRAM bytes per pattern of the float32 training kernel on the 203-120-26
-# workload: 15,513,856 bytes (15,293,952 read + 219,904 written) in one ncu
-# capture of the timed k_train launch of `bench.py --patterns 16384` (16,384
-# patterns after an L2 flush; profiles/k_train_nettalk120_launches.md).  The
-# inputs and targets are read once (916 bytes per pattern); everything else
-# stays in L2.  Re-measure after any change to the kernel.
-K_TRAIN_DRAM_BYTES_PER_PATTERN = 15_513_856 / 16_384
+def cpu_baselines(name, minibatch, patterns, one_core, all_cores, label):
+    """{value, unit, cores, kind, sample, one_core} for a workload: the serial
+    oracle on one core (one_core) and the all-core schemes given; value and
+    cores are those of the fastest."""
+    W = connections(synth_sizes(name))
+    r1 = time_cpu(dict(one_core, workload=name, minibatch=minibatch, patterns=patterns))
+    out = {"value": None, "unit": UNIT, "cores": None, "kind": "oracle",
+           "one_core": W * r1["patterns"] / r1["seconds"]}
+    best = None
+    for spec in all_cores:
+        r = time_cpu(dict(spec, workload=name, minibatch=minibatch, patterns=patterns))
+        v = W * r["patterns"] / r["seconds"]
+        if best is None or v > best[0]:
+            best = (v, r, spec["mode"])
+    if best is None or best[0] < out["one_core"]:
+        # the exchange per group costs more than it saves at this group size
+        out.update(value=out["one_core"], cores=1,
+                   sample=f"{label}; serial on one core, {r1['patterns']} patterns in "
+                          f"{r1['seconds']:.1f} s" + ("" if best is None else
+                                                      f"; {best[2]} on {best[1]['cores']} "
+                                                      f"cores slower ({best[0]:.3g})"))
+    else:
+        out.update(value=best[0], cores=best[1]["cores"],
+                   sample=f"{label}; {best[2]} on {best[1]['cores']} cores, "
+                          f"{best[1]['patterns']} patterns in {best[1]['seconds']:.1f} s")
+    return out
+
+
+def synth_sizes(name):
+    from paper_1801_01554_gb300 import synth
+    return synth.WORKLOADS[name]["sizes"]
+
+
+# DRAM bytes (read + write) per pattern of the dominant kernel of each workload,
+# from single-pass ncu captures (dram__bytes_read.sum + dram__bytes_write.sum)
+# summarised under profiles/, or None until the current kernels are captured.
+TRAFFIC_PER_PATTERN = {
+    "nettalk60": None,
+    "nettalk120": None,
+    "wide3": None,
+    "wide4096": None,
+}
 
 
 def connections(sizes):
@@ -221,6 +289,16 @@ def measured_peaks():
         return {}
 
 
+def alu_peak_tflops(num_sms):
+    sm_max = float(measured_peaks().get("sm_max_mhz", SM_MAX_MHZ_NOMINAL))
+    return num_sms * FP32_LANES_PER_SM * 2 * sm_max * 1e6 / 1e12, sm_max
+
+
+def bf16_peak_tflops():
+    p = measured_peaks().get("bf16_tflops")
+    return (float(p), "measured bf16 cuBLAS, burst") if p else (1900.0, "fallback bf16 burst")
+
+
 # ------------------------------------------------------------------ reference arm
 def run_reference(args, world, rank):
     if rank != 0:
@@ -230,9 +308,13 @@ def run_reference(args, world, rank):
     sizes = w["sizes"]
     W = connections(sizes)
     sample = 4096                      # 8 updates of 512 patterns per step
-    runs = time_oracle(sample, 60.0, steps=args.steps, warmup=args.warmup)
-    tot_p = sum(r["patterns"] for r in runs)
-    tot_s = sum(r["seconds"] for r in runs)
+    tot_p = tot_s = 0.0
+    for k in range(args.warmup + args.steps):
+        r = time_cpu({"mode": "serial", "workload": WORKLOAD, "minibatch": w["minibatch"],
+                      "patterns": sample, "min_s": 0.0, "max_s": 60.0})
+        if k >= args.warmup:
+            tot_p += r["patterns"]
+            tot_s += r["seconds"]
     cps = W * tot_p / tot_s
     line = {
         "impl": "reference", "metric": METRIC, "value": cps, "unit": UNIT, "n_gpus": args.gpus,
@@ -242,16 +324,175 @@ def run_reference(args, world, rank):
         "config": {"workload": workload_desc(w), "global_batch": w["minibatch"],
                    "patterns_per_step": sample, "parallelism": "none (host oracle)"},
         "cpu_baseline": {"value": cps, "unit": UNIT, "cores": 1, "kind": "oracle",
-                         "sample": f"{sample} patterns (8 updates of 512) of the workload per "
-                                   "step, float64 numpy oracle, one BLAS thread"},
+                         "sample": f"{sample} patterns (8 updates of 512) per step, float64 numpy "
+                                   "oracle, one BLAS thread"},
         "e2e": {"value": cps, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
     }
     print(json.dumps(line), flush=True)
     return 0
 
 
-# ------------------------------------------------------------------ our arm
+# ------------------------------------------------------------------ our arm: pieces
+def _events(n):
+    import torch
+    return [torch.cuda.Event(enable_timing=True) for _ in range(n)]
+
+
+def time_f32_launches(net, Xd, Td, n, mb, launches, steps, warmup, flush, stream, sse):
+    """`steps` timed steps of `launches` epoch launches each (L2 flushed before
+    every step).  Returns (per-step ms, per-launch ms)."""
+    import torch
+    for _ in range(warmup):
+        for _ in range(launches):
+            net.train_epoch(Xd, Td, n, mb, sse, stream)
+    net.check(stream)
+    ev = [_events(launches + 1) for _ in range(steps)]
+    torch.cuda.synchronize()
+    for k in range(steps):
+        flush.fill_(float(k))
+        ev[k][0].record(stream)
+        for e in range(launches):
+            net.train_epoch(Xd, Td, n, mb, sse, stream)
+            ev[k][e + 1].record(stream)
+    torch.cuda.synchronize()
+    net.check(stream)
+    step_ms = [ev[k][0].elapsed_time(ev[k][-1]) for k in range(steps)]
+    launch_ms = [ev[k][e].elapsed_time(ev[k][e + 1]) for k in range(steps) for e in range(launches)]
+    return step_ms, launch_ms
+
+
+def time_f32_e2e(net, X, T, n, mb, launches, steps, stream, world, device):
+    """The same steps through bp_train_epoch_host on pinned host buffers: the
+    copies in and the error sums out are inside the timed region."""
+    import torch
+    Xh = torch.tensor(X, dtype=torch.float32).pin_memory()
+    Th = torch.tensor(T, dtype=torch.float32).pin_memory()
+    sse_h = np.zeros(-(-n // mb), dtype=np.float32)
+    net.train_epoch_host(Xh, Th, n, mb, sse_h, stream)      # staging allocation, untimed
+    barrier(world)
+    torch.cuda.synchronize(device)
+    t0 = time.perf_counter()
+    for _ in range(steps):
+        for _ in range(launches):
+            net.train_epoch_host(Xh, Th, n, mb, sse_h, stream)
+    t = allreduce_max(time.perf_counter() - t0, world, device)
+    return t, launches * int(Xh.numel() * 4 + Th.numel() * 4), launches * int(sse_h.nbytes)
+
+
+def f32_entry(name, sizes, n, mb, launches, step_ms, launch_ms, e2e, num_sms, cpu, label):
+    """Compact config entry of a float32 workload."""
+    W = connections(sizes)
+    step_s = sum(step_ms) / len(step_ms) / 1e3
+    launch_s = sum(launch_ms) / len(launch_ms) / 1e3
+    peak, _ = alu_peak_tflops(num_sms)
+    achieved = algorithmic_flops_per_pattern(sizes) * n / launch_s / 1e12
+    tr = TRAFFIC_PER_PATTERN.get(name)
+    ent = {"workload": label, "value": W * n * launches / step_s, "ms_per_step": 1e3 * step_s,
+           "roofline": {"bound": "alu", "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
+                        "frac": achieved / peak, "traffic": tr * n if tr else None}}
+    if e2e is not None:
+        t, bi, bo = e2e[0], e2e[1], e2e[2]
+        ent["e2e"] = {"value": W * n * launches * e2e[3] / t, "unit": UNIT,
+                      "h2d_bytes_per_step": bi, "d2h_bytes_per_step": bo}
+    if cpu is not None:
+        ent["cpu_baseline"] = cpu
+    return ent
+
+
+def bf16_entry(name, sizes, B, step_ms, e2e, cpu, label):
+    W = connections(sizes)
+    step_s = sum(step_ms) / len(step_ms) / 1e3
+    peak, basis = bf16_peak_tflops()
+    achieved = algorithmic_flops_per_pattern(sizes) * B / step_s / 1e12
+    tr = TRAFFIC_PER_PATTERN.get(name)
+    ent = {"workload": label, "value": W * B / step_s, "ms_per_step": 1e3 * step_s,
+           "roofline": {"bound": "tensor", "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
+                        "frac": achieved / peak, "traffic": tr * B if tr else None,
+                        "peak_basis": basis}}
+    if e2e is not None:
+        t, bi, bo, steps = e2e
+        ent["e2e"] = {"value": W * B * steps / t, "unit": UNIT, "h2d_bytes_per_step": bi,
+                      "d2h_bytes_per_step": bo}
+    if cpu is not None:
+        ent["cpu_baseline"] = cpu
+    return ent
+
+
+def measure_bf16(name, steps, warmup, stream, device, world, with_e2e=True):
+    """One bench step = one training update of the full batch (bp_train_batch);
+    `steps` updates back to back, each timed with CUDA events."""
+    import torch
+    from paper_1801_01554_gb300 import bp, synth
+    w = synth.WORKLOADS[name]
+    sizes, X, T, theta = synth.make_workload(name)
+    B = w["minibatch"]
+    Xh = torch.tensor(X, dtype=torch.float32).to(torch.bfloat16)
+    Th = torch.tensor(T, dtype=torch.float32).to(torch.bfloat16)
+    del X, T
+    Xd, Td = Xh.to(device), Th.to(device)
+    sse = torch.zeros(1, dtype=torch.float32, device=device)
+    with bp.Net(sizes, w["lr"], w["momentum"], bp.BP_BF16, max_batch=B) as net:
+        net.set_weights(theta)
+        for _ in range(warmup):
+            net.train_batch(Xd, Td, B, sse, stream)
+        net.check(stream)
+        ev = _events(steps + 1)
+        torch.cuda.synchronize(device)
+        ev[0].record(stream)
+        for k in range(steps):
+            net.train_batch(Xd, Td, B, sse, stream)
+            ev[k + 1].record(stream)
+        torch.cuda.synchronize(device)
+        net.check(stream)
+        step_ms = [ev[k].elapsed_time(ev[k + 1]) for k in range(steps)]
+        e2e = None
+        if with_e2e:
+            Xp, Tp = Xh.pin_memory(), Th.pin_memory()
+            sse_h = np.zeros(1, dtype=np.float32)
+            net.train_epoch_host(Xp, Tp, B, B, sse_h, stream)       # staging allocation
+            e2e_steps = max(1, min(steps, 10))
+            barrier(world)
+            torch.cuda.synchronize(device)
+            t0 = time.perf_counter()
+            for _ in range(e2e_steps):
+                net.train_epoch_host(Xp, Tp, B, B, sse_h, stream)
+            t = allreduce_max(time.perf_counter() - t0, world, device)
+            e2e = (t, int(Xp.numel() * 2 + Tp.numel() * 2), int(sse_h.nbytes), e2e_steps)
+    return sizes, B, step_ms, e2e
+
+
+WIDE_LABEL = {"wide3": "1024-2048-2048-512 bf16, batch 8,192, lr 0.01, m 0.9; step = 1 update",
+              "wide4096": "4096^5 bf16, batch 16,384, lr 0.01, m 0.9; step = 1 update"}
+F32_LABEL = {"nettalk60": "203-60-26 f32, 1,024 patterns, full batch, lr 0.1; step = 10 epochs",
+             "nettalk120": "203-120-26 f32, 65,536 patterns, mb 512, lr 0.05; step = 5 epochs"}
+
+
+def cpu_for(name, mb=None, patterns=None, quick=False, seconds=10.0):
+    """CPU baselines of a workload (bounded samples; see _cpu_child)."""
+    from paper_1801_01554_gb300 import synth
+    w = synth.WORKLOADS[name]
+    ncpu = os.cpu_count() or 1
+    if name in ("wide3", "wide4096"):
+        # one full group of the 1024-2048-2048-512 net; one group of 1,024 of the
+        # 4096^5 net (its 16,384 would take minutes on one core); CPS per pattern
+        B = w["minibatch"] if name == "wide3" else 1024
+        return cpu_baselines(name, B, B, {"mode": "serial", "groups": 1},
+                             [{"mode": "blas", "groups": 1}],
+                             f"one update of {B} patterns, numpy float64 oracle")
+    mb = mb or w["minibatch"]
+    n = patterns or w["patterns"]
+    s1 = 2.0 if quick else seconds
+    specs = []
+    if mb >= 64:
+        specs.append({"mode": "case_parallel", "workers": ncpu, "min_s": s1 / 2, "max_s": 2 * s1})
+    return cpu_baselines(name, mb, n, {"mode": "serial", "min_s": s1, "max_s": 6 * s1}, specs,
+                         f"groups of {mb} of {n} patterns, numpy float64 oracle")
+
+
 def run_ours(args, world, rank, local):
+    """Headline: the 203-120-26 workload, one step = its 5 epochs (5 persistent
+    launches); `configs`: the other workloads, each with its own roofline,
+    CPU baseline and end-to-end figure."""
     import torch
     from paper_1801_01554_gb300 import bp, synth
 
@@ -259,39 +500,39 @@ def run_ours(args, world, rank, local):
         raise SystemExit("bench.py needs a CUDA GPU")
     torch.cuda.set_device(local)
     device = torch.device("cuda", local)
-    w = synth.WORKLOADS[args.workload]
-    sizes, X, T, theta = synth.make_workload(args.workload, patterns=args.patterns)
+    stream = torch.cuda.current_stream(device)
+    num_sms = torch.cuda.get_device_properties(device).multi_processor_count
+    lead = rank == 0 and world == 1 and not args.no_cpu_baseline
+
+    # CPU baselines first, each in its own interpreter (no GPU work running)
+    cpu = {}
+    if lead:
+        cpu["nettalk120"] = cpu_for("nettalk120", patterns=args.patterns, seconds=args.cpu_seconds)
+        if not args.headline_only:
+            cpu["nettalk60"] = cpu_for("nettalk60", quick=True)
+            for B in synth.SWEEP_BATCHES:
+                n = 65536 if B >= 512 else B * 512
+                cpu[("sweep", B)] = cpu_for("nettalk120", mb=B, patterns=n, quick=True)
+            cpu["wide3"] = cpu_for("wide3")
+            cpu["wide4096"] = cpu_for("wide4096")
+
+    flush = torch.empty(L2_FLUSH_BYTES // 4, dtype=torch.float32, device=device)
+    w = synth.WORKLOADS[WORKLOAD]
+    sizes, X, T, theta = synth.make_workload(WORKLOAD, patterns=args.patterns)
     n, mb = len(X), w["minibatch"]
-    updates = (n + mb - 1) // mb
+    epochs = w["epochs"]
+    updates = -(-n // mb)
     W = connections(sizes)
-
-    # CPU baseline first (before any GPU work in this process is irrelevant: it
-    # runs in its own interpreter), on rank 0 only, single-GPU runs only.
-    cpu = None
-    if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        # whole epochs until at least --cpu-seconds of CPU work (60 s cap)
-        r = time_oracle(n, 60.0, min_s=args.cpu_seconds, max_epochs=10 ** 6,
-                        workload=args.workload)[0]
-        cpu = {"value": W * r["patterns"] / r["seconds"], "unit": UNIT, "cores": 1,
-               "kind": "oracle",
-               "sample": f"{r['patterns']} patterns ({r['patterns'] / n:.2f} epochs of the "
-                         f"workload, {(r['patterns'] + mb - 1) // mb} updates of {mb}), float64 "
-                         f"numpy oracle, one BLAS thread, {r['seconds']:.1f} s"}
-
     Xd = torch.tensor(X, dtype=torch.float32, device=device)
     Td = torch.tensor(T, dtype=torch.float32, device=device)
     sse = torch.zeros(updates, dtype=torch.float32, device=device)
-    flush = torch.empty(L2_FLUSH_BYTES // 4, dtype=torch.float32, device=device)
-    stream = torch.cuda.current_stream(device)
-
     net = bp.Net(sizes, w["lr"], w["momentum"], bp.BP_F32, max_batch=mb)
     net.set_weights(theta)
     for _ in range(args.warmup):
-        net.train_epoch(Xd, Td, n, mb, sse, stream)
+        for _ in range(epochs):
+            net.train_epoch(Xd, Td, n, mb, sse, stream)
     net.check(stream)
-
-    starts = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
-    ends = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+    ev = [_events(epochs + 1) for _ in range(args.steps)]
     clocks = ClockSampler(local)
     barrier(world)
     torch.cuda.synchronize(device)
@@ -299,142 +540,109 @@ def run_ours(args, world, rank, local):
     time.sleep(0.3)   # let the sampler start before the timed region
     t_wall0 = time.perf_counter()
     for k in range(args.steps):
-        flush.fill_(float(k))                  # evict the previous epoch from L2
-        starts[k].record(stream)
-        net.train_epoch(Xd, Td, n, mb, sse, stream)
-        ends[k].record(stream)
+        flush.fill_(float(k))                  # evict the previous step from L2
+        ev[k][0].record(stream)
+        for e in range(epochs):
+            net.train_epoch(Xd, Td, n, mb, sse, stream)
+            ev[k][e + 1].record(stream)
     torch.cuda.synchronize(device)
     t_wall = time.perf_counter() - t_wall0
     clk = clocks.stop()
     barrier(world)
     net.check(stream)
-    per_step_ms = [s.elapsed_time(e) for s, e in zip(starts, ends)]
-    dev_s = sum(per_step_ms) / 1e3
+    step_ms = [ev[k][0].elapsed_time(ev[k][-1]) for k in range(args.steps)]
+    launch_ms = [ev[k][e].elapsed_time(ev[k][e + 1]) for k in range(args.steps) for e in range(epochs)]
+    dev_s = sum(step_ms) / 1e3
     dev_s_max = allreduce_max(dev_s, world, device)
-    patterns_all = n * args.steps * world
-    value = W * patterns_all / dev_s_max
-
-    # end to end: host buffers through bp_train_epoch_host, copies inside the timed region
-    Xh = torch.tensor(X, dtype=torch.float32).pin_memory()
-    Th = torch.tensor(T, dtype=torch.float32).pin_memory()
-    sse_h = np.zeros(updates, dtype=np.float32)
-    e2e_steps = max(1, min(args.steps, 20))
-    net.train_epoch_host(Xh, Th, n, mb, sse_h, stream)     # staging allocation, untimed
-    barrier(world)
-    torch.cuda.synchronize(device)
-    t0 = time.perf_counter()
-    for _ in range(e2e_steps):
-        net.train_epoch_host(Xh, Th, n, mb, sse_h, stream)
-    e2e_s = allreduce_max(time.perf_counter() - t0, world, device)
-    e2e_value = W * n * e2e_steps * world / e2e_s
+    value = W * n * epochs * args.steps * world / dev_s_max
+    e2e_steps = max(1, min(args.steps, 10))
+    t_e2e, bi, bo = time_f32_e2e(net, X, T, n, mb, epochs, e2e_steps, stream, world, device)
     net.close()
 
-    # roofline of the training kernel: algorithmic flops / FFMA peak
-    flops_launch = algorithmic_flops_per_pattern(sizes) * n
-    kernel_s = dev_s / args.steps
-    achieved = flops_launch / kernel_s / 1e12
-    peaks = measured_peaks()
-    sm_max = float(peaks.get("sm_max_mhz", SM_MAX_MHZ_NOMINAL))
-    num_sms = torch.cuda.get_device_properties(device).multi_processor_count
-    peak = num_sms * FP32_LANES_PER_SM * 2 * sm_max * 1e6 / 1e12
-
+    launch_s = sum(launch_ms) / len(launch_ms) / 1e3
+    peak, sm_max = alu_peak_tflops(num_sms)
+    achieved = algorithmic_flops_per_pattern(sizes) * n / launch_s / 1e12
+    tr = TRAFFIC_PER_PATTERN[WORKLOAD] if args.patterns is None else None
     line = {
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": 1e3 * dev_s_max / args.steps,
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32",
         "data": "synthetic",
-        "config": {"workload": workload_desc(w), "global_batch": mb,
-                   "patterns_per_step": n, "updates_per_step": updates,
+        "config": {"workload": F32_LABEL[WORKLOAD], "global_batch": mb,
+                   "patterns_per_step": n * epochs, "updates_per_step": updates * epochs,
                    "parallelism": "replicas" if world > 1 else "single GPU",
-                   "l2": f"flushed ({L2_FLUSH_BYTES >> 20} MB write) before every timed epoch; "
-                         "an epoch reads each pattern once"},
+                   "l2": "flushed (512 MB write) before every timed step"},
         "roofline": {"bound": "alu", "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
-                     "frac": achieved / peak,
-                     "traffic": K_TRAIN_DRAM_BYTES_PER_PATTERN * n if args.workload == WORKLOAD
-                     else None,
-                     "traffic_basis": "ncu dram__bytes_read.sum + dram__bytes_write.sum of the "
-                                      "timed k_train launch of bench.py --patterns 16384 (after "
-                                      "an L2 flush), scaled to the launch's patterns",
-                     "kernel": "k_train (persistent cooperative training kernel)",
-                     "peak_basis": f"{num_sms} SMs x {FP32_LANES_PER_SM} FP32 lanes x 2 flop x "
+                     "frac": achieved / peak, "traffic": tr * n if tr else None,
+                     "kernel": "k_train, one launch per epoch (CUDA events per launch)",
+                     "peak_basis": f"{num_sms} SMs x {FP32_LANES_PER_SM} FFMA lanes x 2 x "
                                    f"{sm_max:.0f} MHz"},
-        "e2e": {"value": e2e_value, "unit": UNIT,
-                "h2d_bytes_per_step": int(Xh.numel() * 4 + Th.numel() * 4),
-                "d2h_bytes_per_step": int(sse_h.nbytes)},
-        "gpu_launches": args.steps,
+        "e2e": {"value": W * n * epochs * e2e_steps * world / t_e2e, "unit": UNIT,
+                "h2d_bytes_per_step": bi, "d2h_bytes_per_step": bo},
+        "gpu_launches": args.steps * epochs,
         "clocks": clk,
         "wall_s_timed": t_wall,
     }
-    if cpu is not None:
-        line["cpu_baseline"] = cpu
+    if "nettalk120" in cpu:
+        line["cpu_baseline"] = cpu["nettalk120"]
+
+    if not args.headline_only:
+        configs = {}
+        # 203-60-26: one step = its 10 epochs of one full-batch update each
+        w0 = synth.WORKLOADS["nettalk60"]
+        s0, X0, T0, th0 = synth.make_workload("nettalk60")
+        n0 = len(X0)
+        with bp.Net(s0, w0["lr"], w0["momentum"], bp.BP_F32, max_batch=n0) as net0:
+            net0.set_weights(th0)
+            X0d = torch.tensor(X0, dtype=torch.float32, device=device)
+            T0d = torch.tensor(T0, dtype=torch.float32, device=device)
+            sse0 = torch.zeros(1, device=device)
+            sm, lm = time_f32_launches(net0, X0d, T0d, n0, n0, w0["epochs"], 20, args.warmup, flush,
+                                       stream, sse0)
+            e = time_f32_e2e(net0, X0, T0, n0, n0, w0["epochs"], 10, stream, world, device)
+        configs["nettalk60"] = f32_entry("nettalk60", s0, n0, n0, w0["epochs"], sm, lm,
+                                         (e[0], e[1], e[2], 10), num_sms, cpu.get("nettalk60"),
+                                         F32_LABEL["nettalk60"])
+        # group-size sweep on 203-120-26: one step = one epoch
+        sweep = []
+        for B in synth.SWEEP_BATCHES:
+            nb = 65536 if B >= 512 else B * 512
+            with bp.Net(sizes, w["lr"], w["momentum"], bp.BP_F32, max_batch=B) as netb:
+                netb.set_weights(theta)
+                sseb = torch.zeros(-(-nb // B), device=device)
+                sm, lm = time_f32_launches(netb, Xd, Td, nb, B, 1, 5, 3, flush, stream, sseb)
+                e = time_f32_e2e(netb, X[:nb], T[:nb], nb, B, 1, 3, stream, world, device)
+            ent = f32_entry("sweep", sizes, nb, B, 1, sm, lm, (e[0], e[1], e[2], 3), num_sms,
+                            None, "")
+            c = cpu.get(("sweep", B))
+            sweep.append({"B": B, "patterns": nb, "value": ent["value"],
+                          "us_per_update": 1e3 * ent["ms_per_step"] / -(-nb // B),
+                          "frac": ent["roofline"]["frac"], "e2e": ent["e2e"]["value"],
+                          "cpu_one_core": c["one_core"] if c else None,
+                          "cpu_all_cores": c["value"] if c else None,
+                          "cpu_cores": c["cores"] if c else None})
+        configs["sweep_nettalk120"] = sweep
+        for name in ("wide3", "wide4096"):
+            steps = synth.WORKLOADS[name]["steps"]
+            sz, B, sm, e = measure_bf16(name, steps, args.warmup, stream, device, world)
+            configs[name] = bf16_entry(name, sz, B, sm, e, cpu.get(name), WIDE_LABEL[name])
+        line["configs"] = configs
     if rank == 0:
         print(json.dumps(line), flush=True)
     return 0
 
 
 def run_wide(args, world, rank, local):
-    """BF16 tensor-core workloads: one step = one training update on the full batch."""
+    """One bf16 workload alone (for profiler captures): its compact entry."""
     import torch
-    from paper_1801_01554_gb300 import bp, synth
-
     torch.cuda.set_device(local)
     device = torch.device("cuda", local)
-    name = args.workload
-    w = synth.WORKLOADS[name]
-    sizes, X, T, theta = synth.make_workload(name)
-    B = w["minibatch"]
-    W = connections(sizes)
-    Xd = torch.tensor(X, dtype=torch.float32, device=device).to(torch.bfloat16)
-    Td = torch.tensor(T, dtype=torch.float32, device=device).to(torch.bfloat16)
-    del X, T
-    sse = torch.zeros(1, dtype=torch.float32, device=device)
     stream = torch.cuda.current_stream(device)
-    net = bp.Net(sizes, w["lr"], w["momentum"], bp.BP_BF16, max_batch=B)
-    net.set_weights(theta)
-    for _ in range(args.warmup):
-        net.train_batch(Xd, Td, B, sse, stream)
-    net.check(stream)
-    starts = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
-    ends = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
-    clocks = ClockSampler(local)
-    barrier(world)
-    torch.cuda.synchronize(device)
-    clocks.start()
-    time.sleep(0.3)
-    for k in range(args.steps):
-        starts[k].record(stream)
-        net.train_batch(Xd, Td, B, sse, stream)
-        ends[k].record(stream)
-    torch.cuda.synchronize(device)
-    clk = clocks.stop()
-    net.check(stream)
-    dev_s = sum(s_.elapsed_time(e_) for s_, e_ in zip(starts, ends)) / 1e3
-    dev_s_max = allreduce_max(dev_s, world, device)
-    value = W * B * args.steps * world / dev_s_max
-    flops = algorithmic_flops_per_pattern(sizes) * B
-    achieved = flops / (dev_s / args.steps) / 1e12
-    peaks = measured_peaks()
-    peak = float(peaks.get("bf16_tflops_sustained", 1700.0))
-    net.close()
-    line = {
-        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
-        "warmup": args.warmup, "ms_per_step": 1e3 * dev_s_max / args.steps,
-        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
-        "data": "synthetic",
-        "config": {"workload": f"{'-'.join(map(str, sizes))} sigmoid MLP, bf16 activations and "
-                               f"weight copies, fp32 accumulate and master weights, batch {B}, "
-                               f"lr {w['lr']}, momentum {w['momentum']}; one step = one update",
-                   "global_batch": B, "parallelism": "single GPU",
-                   "l2": "activations of one step exceed the 129 MB L2"},
-        "roofline": {"bound": "tensor", "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
-                     "frac": achieved / peak, "traffic": None,
-                     "kernel": "whole training step (k_gemm forward, hidden-delta and pooled-change "
-                               "GEMMs, transposes, update); flops = (6W - 2W_i) per pattern",
-                     "peak_basis": "measured bf16 cuBLAS, sustained"},
-        "clocks": clk,
-    }
+    sz, B, sm, e = measure_bf16(args.workload, args.steps, args.warmup, stream, device, world,
+                                with_e2e=False)
     if rank == 0:
-        print(json.dumps(line), flush=True)
+        print(json.dumps({args.workload: bf16_entry(args.workload, sz, B, sm, e, None,
+                                                    WIDE_LABEL[args.workload])}), flush=True)
     return 0
 
 
@@ -540,11 +748,15 @@ def main():
     ap.add_argument("--steps", type=int, default=200)
     ap.add_argument("--warmup", type=int, default=10)
     ap.add_argument("--impl", choices=("ours", "reference"), default="ours")
-    ap.add_argument("--cpu-seconds", type=float, default=10.0)
+    ap.add_argument("--cpu-seconds", type=float, default=10.0,
+                    help="one-core oracle seconds for the headline workload's CPU baseline")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--workload", default=WORKLOAD,
-                    choices=("nettalk60", "nettalk120", "wide3", "wide4096"),
-                    help="workload to time (default: the 203-120-26 NETtalk-shaped net)")
+                    choices=("nettalk120", "wide3", "wide4096"),
+                    help="nettalk120 (default): the headline and every config; wide3/wide4096: "
+                         "that bf16 workload alone, for profiler captures")
+    ap.add_argument("--headline-only", action="store_true",
+                    help="the 203-120-26 headline alone (no configs object)")
     ap.add_argument("--patterns", type=int, default=None,
                     help="patterns per epoch (default: the workload's; a smaller epoch of the "
                          "same net and group size is for profiler captures, not a bench line)")
@@ -555,6 +767,8 @@ def main():
     args = ap.parse_args()
     if args.warmup < 3 and args.impl == "ours":
         args.warmup = 3
+    if args.patterns is not None:
+        args.headline_only = True      # a shortened epoch is for profiler captures only
     world, rank, local = dist_setup()
     if args.impl == "reference":
         rc = run_reference(args, world, rank)
