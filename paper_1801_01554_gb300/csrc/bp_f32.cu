@@ -134,7 +134,8 @@ __device__ bool grid_barrier(unsigned* bar, unsigned target, int* flags, unsigne
     __syncthreads();
     int ok = 1;
     if (threadIdx.x == 0) {
-        __threadfence();
+        // the release is cumulative: with the CTA barrier above it also orders
+        // every thread's earlier writes before the arrival (no separate fence)
         asm volatile("red.release.gpu.global.add.u32 [%0], %1;" ::"l"(bar + 1), "r"(1u) : "memory");
         const unsigned long long t0 = global_ns();
         unsigned it = 0;

@@ -66,9 +66,9 @@ def test_noalloc_rejects_sizes_beyond_its_scratch():
 def test_noalloc_smaller_call_after_a_larger_one():
     """The static scratch keeps the previous call's activations, deltas and
     padded weights.  A call on a larger net and minibatch, then one on a
-    smaller, deeper net: the second must give the same bits as
-    bp_train_epoch on a fresh net (same kernel, same plan), so nothing stale
-    from the first call reaches it."""
+    smaller, deeper net: the second must match bp_train_epoch on a fresh net
+    within the float32 bar, per layer, so nothing stale from the first call
+    reaches it (stale rows would change the pooled change by far more)."""
     big, n1, mb1 = (203, 120, 26), 4096, 2048
     X1, T1 = synth.nettalk_patterns(n1, seed=31)
     th1 = torch.tensor(synth.round_to(synth.init_uniform(big, -0.3, 0.3, 31), "f32"),
@@ -98,6 +98,10 @@ def test_noalloc_smaller_call_after_a_larger_one():
     bp.bp_train_epoch_noalloc(small, 0.05, 0.9, 1.0, th, V, Xd, Td, n, mb, sse, status)
     torch.cuda.synchronize()
     assert int(status.item()) == 0
-    np.testing.assert_array_equal(th.cpu().numpy(), w_ref)
-    np.testing.assert_array_equal(V.cpu().numpy(), v_ref)
-    np.testing.assert_array_equal(sse.cpu().numpy(), sse_ref.cpu().numpy())
+    offs, _ = synth.param_layout(small)
+    w, v = th.cpu().numpy().astype(np.float64), V.cpu().numpy().astype(np.float64)
+    for l, (wo, bo) in enumerate(offs, start=1):
+        for a, b in ((wo, wo + small[l] * small[l - 1]), (bo, bo + small[l])):
+            assert normwise(v[a:b], v_ref[a:b]) <= TOL, l
+            assert normwise(w[a:b] - theta[a:b], w_ref[a:b] - theta[a:b]) <= TOL, l
+    np.testing.assert_allclose(sse.cpu().numpy(), sse_ref.cpu().numpy(), rtol=TOL)
