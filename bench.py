@@ -259,14 +259,18 @@ def synth_sizes(name):
     return synth.WORKLOADS[name]["sizes"]
 
 
-# DRAM bytes (read + write) per pattern of the dominant kernel of each workload,
-# from single-pass ncu captures (dram__bytes_read.sum + dram__bytes_write.sum)
-# summarised under profiles/, or None until the current kernels are captured.
+# DRAM bytes (read + write) per pattern of each workload's roofline unit, from
+# single-pass ncu captures (dram__bytes_read.sum + dram__bytes_write.sum; the
+# commands are in profiles/dram_traffic_all_workloads.md): one k_train launch
+# for the float32 nets (one epoch; 203-120-26 captured on a 16,384-pattern epoch
+# and scaled by patterns, as its traffic is the inputs read once), the whole
+# training step (all launches) for the bf16 nets.  Re-measure after any change
+# to these kernels.
 TRAFFIC_PER_PATTERN = {
-    "nettalk60": None,
-    "nettalk120": None,
-    "wide3": None,
-    "wide4096": None,
+    "nettalk60": 1_124_864 / 1024,          # 1.12 MB per launch (one update of 1,024)
+    "nettalk120": 15_532_288 / 16384,       # 62.1 MB per 65,536-pattern launch
+    "wide3": 585_467_136 / 8192,            # 585 MB per step
+    "wide4096": 9_221_444_864 / 16384,      # 9.22 GB per step
 }
 
 
@@ -632,6 +636,32 @@ def run_ours(args, world, rank, local):
     return 0
 
 
+def run_nettalk60(args, world, rank, local):
+    """The 203-60-26 workload alone (for profiler captures): its compact entry;
+    one step = its 10 full-batch epochs, one launch each."""
+    import torch
+    from paper_1801_01554_gb300 import bp, synth
+    torch.cuda.set_device(local)
+    device = torch.device("cuda", local)
+    stream = torch.cuda.current_stream(device)
+    num_sms = torch.cuda.get_device_properties(device).multi_processor_count
+    flush = torch.empty(L2_FLUSH_BYTES // 4, dtype=torch.float32, device=device)
+    w0 = synth.WORKLOADS["nettalk60"]
+    s0, X0, T0, th0 = synth.make_workload("nettalk60")
+    n0 = len(X0)
+    with bp.Net(s0, w0["lr"], w0["momentum"], bp.BP_F32, max_batch=n0) as net0:
+        net0.set_weights(th0)
+        X0d = torch.tensor(X0, dtype=torch.float32, device=device)
+        T0d = torch.tensor(T0, dtype=torch.float32, device=device)
+        sse0 = torch.zeros(1, device=device)
+        sm, lm = time_f32_launches(net0, X0d, T0d, n0, n0, w0["epochs"], args.steps, args.warmup,
+                                   flush, stream, sse0)
+    if rank == 0:
+        print(json.dumps({"nettalk60": f32_entry("nettalk60", s0, n0, n0, w0["epochs"], sm, lm, None,
+                                                 num_sms, None, F32_LABEL["nettalk60"])}), flush=True)
+    return 0
+
+
 def run_wide(args, world, rank, local):
     """One bf16 workload alone (for profiler captures): its compact entry."""
     import torch
@@ -752,9 +782,9 @@ def main():
                     help="one-core oracle seconds for the headline workload's CPU baseline")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--workload", default=WORKLOAD,
-                    choices=("nettalk120", "wide3", "wide4096"),
-                    help="nettalk120 (default): the headline and every config; wide3/wide4096: "
-                         "that bf16 workload alone, for profiler captures")
+                    choices=("nettalk120", "nettalk60", "wide3", "wide4096"),
+                    help="nettalk120 (default): the headline and every config; nettalk60, wide3, "
+                         "wide4096: that workload alone, for profiler captures")
     ap.add_argument("--headline-only", action="store_true",
                     help="the 203-120-26 headline alone (no configs object)")
     ap.add_argument("--patterns", type=int, default=None,
@@ -778,6 +808,8 @@ def main():
         rc = run_crossover(args, world, rank, local)
     elif args.workload in ("wide3", "wide4096"):
         rc = run_wide(args, world, rank, local)
+    elif args.workload == "nettalk60":
+        rc = run_nettalk60(args, world, rank, local)
     else:
         rc = run_ours(args, world, rank, local)
     if world > 1:
