@@ -55,7 +55,9 @@ constexpr unsigned long long kWaitNs = 2000000000ull;   // 2 s per wait
 constexpr unsigned kWaitIters = 1u << 26;
 
 // ------------------------------------------------------------ small helpers
-__device__ __forceinline__ float sigmoid_f(float x) { return 1.0f / (1.0f + expf(-x)); }
+// Logistic: CUDA's expf and the fast reciprocal divide (2 ulp, far inside the
+// float32 bar; for 1 + e^-x beyond 2^126 the quotient is 0, the logistic's value).
+__device__ __forceinline__ float sigmoid_f(float x) { return __fdividef(1.0f, 1.0f + expf(-x)); }
 
 // Checked build (-DBP_CHECK): phases test that their shared-memory regions fit
 // the launch's dynamic shared memory and that their rows and tile origins lie
@@ -551,13 +553,15 @@ __device__ float pattern_phase(const F32View& v, const PatLayout& q, const float
             return 0.f;
         }
         if (do_fwd) {
+            // the input rows go to scratch first, so that their stores drain during the forward pass
+            if (to_scratch) rows_to_scratch<PG, false>(v, 0, smem + q.sa[0], v.apitch[0], p0, np);
             for (int l = 1; l <= L; ++l) {
                 forward_layer<PG>(Wb + v.woff[l], v.kp[l], v.n[l], smem + q.sa[l - 1], smem + q.sa[l],
                                   v.apitch[l], v.sig_table != 0);
                 __syncthreads();
             }
             // activation rows, bias column and pads included
-            for (int l = 0; l <= L && to_scratch; ++l)
+            for (int l = 1; l <= L && to_scratch; ++l)
                 rows_to_scratch<PG, false>(v, l, smem + q.sa[l], v.apitch[l], p0, np);
             if (Y != nullptr && pr < np) {
                 for (int k = c0; k < nL; k += TP)
