@@ -47,6 +47,7 @@ constexpr int kTJ = 32;           // weight-tile columns (inputs; the bias is th
 constexpr int kPC = 256;          // patterns per staged chunk of the weight phase
 constexpr int kChunkFloats = kPC * (kTU + kTJ);
 constexpr int kNBuf = 3;          // chunk buffers in flight
+constexpr int kWidePG = 32;       // patterns per pass of the whole-row-per-lane forward
 // weight-phase buffers (each chunk: the [kPC][kTJ] activation block, 128-byte
 // swizzled, then the [kPC][kTU] delta block), plus room to align them to 1 KB
 constexpr size_t kGradFloats = kNBuf * kChunkFloats + 256;
@@ -435,6 +436,64 @@ __device__ void forward_layer(const float* W, int kp, int n_out, const float* s_
     }
 }
 
+// Forward through one layer for groups of 32 patterns (PG a multiple of 32):
+// lane p of a warp owns pattern p of its warp's group and sums that pattern's
+// dot products over whole rows for U units at a time, with no cross-lane
+// reduction.  The warps of a group split the units; every lane of a warp reads
+// the same weight float4 (a broadcast), so each activation float4 feeds 4 U
+// FMAs.  The activation rows are read at stride kp: kp / 4 odd keeps the 32
+// lanes' float4 reads at the minimum of four wavefronts (f32_plan checks it).
+template <int PG, int U>
+__device__ void forward_layer_lanes(const float* W, int kp, int n_out, const float* s_in, float* s_out,
+                                    int kp_out, bool table) {
+    static_assert(PG % 32 == 0, "whole warps of patterns");
+    constexpr int kGroups = PG / 32;
+    constexpr int kWarpsPerGroup = kWarps / kGroups;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int p = (warp / kWarpsPerGroup) * 32 + lane, wi = warp % kWarpsPerGroup;
+    const int K4 = kp >> 2;
+    const float* a = s_in + p * kp;
+    for (int j0 = wi * U; j0 < n_out; j0 += kWarpsPerGroup * U) {
+        int wo[U];   // row offsets (rows past the layer repeat its last row)
+#pragma unroll
+        for (int u = 0; u < U; ++u) wo[u] = min(j0 + u, n_out - 1) * kp;
+        float acc[U];
+#pragma unroll
+        for (int u = 0; u < U; ++u) acc[u] = 0.f;
+        for (int k = 0; k < K4; ++k) {
+            const float4 x = ld4(a + 4 * k);
+#pragma unroll
+            for (int u = 0; u < U; ++u) {
+                const float4 w = ld4(W + wo[u] + 4 * k);
+                float t = acc[u];
+                t = fmaf(w.x, x.x, t);
+                t = fmaf(w.y, x.y, t);
+                t = fmaf(w.z, x.z, t);
+                t = fmaf(w.w, x.w, t);
+                acc[u] = t;
+            }
+        }
+#pragma unroll
+        for (int u = 0; u < U; ++u)
+            if (j0 + u < n_out) s_out[p * kp_out + j0 + u] = table ? sigmoid_tab(acc[u]) : sigmoid_f(acc[u]);
+    }
+}
+
+// Forward through one layer for PG patterns held in shared memory: the
+// lane-group form below for small groups, whole rows per lane from 32 up.
+template <int PG>
+__device__ __forceinline__ void forward_any(const float* W, int kp, int n_out, const float* s_in, float* s_out,
+                                            int kp_out, bool table) {
+    if constexpr (PG >= 32) {
+        if (n_out >= 4 * kWarps / (PG / 32))
+            forward_layer_lanes<PG, 8>(W, kp, n_out, s_in, s_out, kp_out, table);
+        else
+            forward_layer_lanes<PG, 2>(W, kp, n_out, s_in, s_out, kp_out, table);
+    } else {
+        forward_layer<PG>(W, kp, n_out, s_in, s_out, kp_out, table);
+    }
+}
+
 // Hidden deltas of layer l for PG patterns: d_l[p][i] = (sum_j W_{l+1}[j][i]
 // d_{l+1}[p][j]) a_l[p][i] (1 - a_l[p][i]), one thread per (pattern, unit)
 // summing over the next layer's units in order.  dnt holds d_{l+1}
@@ -452,6 +511,57 @@ __device__ void hidden_delta(const float* Wn, int kpn, int n, int nn, const floa
         const float d = acc * a * (1.f - a);
         dl[p * dpl + i] = d;
         if (dlt != nullptr) dlt[i * PG + p] = d;
+    }
+}
+
+// Hidden deltas for groups of 32 patterns (PG a multiple of 32): lane p owns
+// pattern p of its warp's group and sums over the next layer's units for U of
+// this layer's units at a time.  The next layer's deltas are read
+// pattern-minor (consecutive lanes, no bank conflict), the weight row pieces
+// W_{l+1}[j][i0 .. i0 + U) as broadcasts.
+template <int PG, int U>
+__device__ void hidden_delta_lanes(const float* Wn, int kpn, int n, int nn, const float* dnt, const float* al,
+                                   int apl, float* dl, int dpl, float* dlt) {
+    static_assert(PG % 32 == 0 && U % 4 == 0, "whole warps of patterns, float4 pieces of rows");
+    constexpr int kGroups = PG / 32;
+    constexpr int kWarpsPerGroup = kWarps / kGroups;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int p = (warp / kWarpsPerGroup) * 32 + lane, wi = warp % kWarpsPerGroup;
+    for (int i0 = wi * U; i0 < n; i0 += kWarpsPerGroup * U) {
+        float acc[U];
+#pragma unroll
+        for (int u = 0; u < U; ++u) acc[u] = 0.f;
+        if (i0 + U <= kpn) {   // the row piece lies inside the padded row
+            for (int j = 0; j < nn; ++j) {
+                const float d = dnt[j * PG + p];
+                const float* wrow = Wn + (size_t)j * kpn + i0;
+#pragma unroll
+                for (int q = 0; q < U / 4; ++q) {
+                    const float4 w = ld4(wrow + 4 * q);
+                    acc[4 * q] = fmaf(d, w.x, acc[4 * q]);
+                    acc[4 * q + 1] = fmaf(d, w.y, acc[4 * q + 1]);
+                    acc[4 * q + 2] = fmaf(d, w.z, acc[4 * q + 2]);
+                    acc[4 * q + 3] = fmaf(d, w.w, acc[4 * q + 3]);
+                }
+            }
+        } else {
+            for (int j = 0; j < nn; ++j) {
+                const float d = dnt[j * PG + p];
+#pragma unroll
+                for (int u = 0; u < U; ++u)
+                    if (i0 + u < n) acc[u] = fmaf(d, Wn[(size_t)j * kpn + i0 + u], acc[u]);
+            }
+        }
+#pragma unroll
+        for (int u = 0; u < U; ++u) {
+            const int i = i0 + u;
+            if (i < n) {
+                const float a = al[p * apl + i];
+                const float dv = acc[u] * a * (1.f - a);
+                dl[p * dpl + i] = dv;
+                if (dlt != nullptr) dlt[i * PG + p] = dv;
+            }
+        }
     }
 }
 
@@ -556,8 +666,8 @@ __device__ float pattern_phase(const F32View& v, const PatLayout& q, const float
             // the input rows go to scratch first, so that their stores drain during the forward pass
             if (to_scratch) rows_to_scratch<PG, false>(v, 0, smem + q.sa[0], v.apitch[0], p0, np);
             for (int l = 1; l <= L; ++l) {
-                forward_layer<PG>(Wb + v.woff[l], v.kp[l], v.n[l], smem + q.sa[l - 1], smem + q.sa[l],
-                                  v.apitch[l], v.sig_table != 0);
+                forward_any<PG>(Wb + v.woff[l], v.kp[l], v.n[l], smem + q.sa[l - 1], smem + q.sa[l],
+                                v.apitch[l], v.sig_table != 0);
                 __syncthreads();
             }
             // activation rows, bias column and pads included
@@ -586,9 +696,14 @@ __device__ float pattern_phase(const F32View& v, const PatLayout& q, const float
             __syncthreads();
             // hidden deltas, output side first; no delta for the input layer
             for (int l = L - 1; l >= 1; --l) {
-                hidden_delta<PG>(Wb + v.woff[l + 1], v.kp[l + 1], v.n[l], v.n[l + 1], smem + q.sdt[l + 1],
-                                 smem + q.sa[l], v.apitch[l], smem + q.sd[l], v.dpitch[l],
-                                 l >= 2 ? smem + q.sdt[l] : nullptr);
+                if constexpr (PG >= 32)
+                    hidden_delta_lanes<PG, 8>(Wb + v.woff[l + 1], v.kp[l + 1], v.n[l], v.n[l + 1],
+                                              smem + q.sdt[l + 1], smem + q.sa[l], v.apitch[l], smem + q.sd[l],
+                                              v.dpitch[l], l >= 2 ? smem + q.sdt[l] : nullptr);
+                else
+                    hidden_delta<PG>(Wb + v.woff[l + 1], v.kp[l + 1], v.n[l], v.n[l + 1], smem + q.sdt[l + 1],
+                                     smem + q.sa[l], v.apitch[l], smem + q.sd[l], v.dpitch[l],
+                                     l >= 2 ? smem + q.sdt[l] : nullptr);
                 __syncthreads();
             }
             for (int l = 1; l <= L && to_scratch; ++l)
@@ -1231,6 +1346,16 @@ int f32_max_pg(const int* n, int L) {
     return best;
 }
 
+// Whether passes of kWidePG patterns (the whole-row-per-lane forward) suit the
+// net: every activation row pitch / 4 odd (conflict-free lane reads) and the
+// weights and pattern buffers together in shared memory.
+static bool wide_pg_ok(const F32View& v) {
+    for (int l = 0; l < v.L; ++l)
+        if (((v.apitch[l] >> 2) & 1) == 0) return false;
+    const size_t need = (size_t)v.wsm + pattern_floats(v.n, v.L, kWidePG);
+    return need * sizeof(float) <= kSmemLimit;
+}
+
 template <int PG, bool GUARD>
 cudaError_t set_small_attr_g(size_t bytes) {
     cudaError_t e = cudaFuncSetAttribute(k_train_small<PG, 4, GUARD>,
@@ -1256,6 +1381,7 @@ cudaError_t f32_setup(int device) {
     if ((e = set_smem_attr<2>(kSmemLimit)) != cudaSuccess) return e;
     if ((e = set_smem_attr<4>(kSmemLimit)) != cudaSuccess) return e;
     if ((e = set_smem_attr<8>(kSmemLimit)) != cudaSuccess) return e;
+    if ((e = set_smem_attr<kWidePG>(kSmemLimit)) != cudaSuccess) return e;
     if ((e = set_small_attr<1>(kSmemLimit)) != cudaSuccess) return e;
     if ((e = set_small_attr<2>(kSmemLimit)) != cudaSuccess) return e;
     if ((e = set_small_attr<4>(kSmemLimit)) != cudaSuccess) return e;
@@ -1269,6 +1395,9 @@ F32Plan f32_plan(const F32View& v, int batch, int num_sms) {
     const int want = (batch + num_sms - 1) / num_sms;
     int pg = 1;
     while (pg < want && pg < maxpg) pg *= 2;
+    // more than 16 patterns per CTA: passes of kWidePG, when the net suits them
+    // (at 9-16 a half-empty pass of 32 is slower than two passes of 8)
+    if (want > 16 && pg == 8 && wide_pg_ok(v)) pg = kWidePG;
     p.pg = pg;
     p.grid = num_sms;
     // weights in shared memory when they fit below the pattern buffers
@@ -1290,7 +1419,8 @@ cudaError_t f32_forward(const F32View& v, const float* X, int batch, float* Y, c
         case 1: BP_FWD(1); break;
         case 2: BP_FWD(2); break;
         case 4: BP_FWD(4); break;
-        default: BP_FWD(8); break;
+        case 8: BP_FWD(8); break;
+        default: BP_FWD(kWidePG); break;
     }
 #undef BP_FWD
     return cudaGetLastError();
@@ -1305,7 +1435,8 @@ cudaError_t f32_backward(const F32View& v, const float* /*X*/, const float* T, i
         case 1: BP_DEL(1); break;
         case 2: BP_DEL(2); break;
         case 4: BP_DEL(4); break;
-        default: BP_DEL(8); break;
+        case 8: BP_DEL(8); break;
+        default: BP_DEL(kWidePG); break;
     }
 #undef BP_DEL
     cudaError_t e = cudaGetLastError();
@@ -1355,7 +1486,8 @@ cudaError_t f32_train(const F32View& v, const float* X, const float* T, int n_pa
         case 1: fn = ws ? (const void*)k_train<1, true> : (const void*)k_train<1, false>; break;
         case 2: fn = ws ? (const void*)k_train<2, true> : (const void*)k_train<2, false>; break;
         case 4: fn = ws ? (const void*)k_train<4, true> : (const void*)k_train<4, false>; break;
-        default: fn = ws ? (const void*)k_train<8, true> : (const void*)k_train<8, false>; break;
+        case 8: fn = ws ? (const void*)k_train<8, true> : (const void*)k_train<8, false>; break;
+        default: fn = ws ? (const void*)k_train<kWidePG, true> : (const void*)k_train<kWidePG, false>; break;
     }
     return cudaLaunchCooperativeKernel(fn, dim3(plan.grid), dim3(kThreads), args, plan.smem, s);
 }
@@ -1424,7 +1556,8 @@ cudaError_t f32_diagnose(const F32View& v, const float* X, const float* T, int b
         case 1: BP_DIAG(1); break;
         case 2: BP_DIAG(2); break;
         case 4: BP_DIAG(4); break;
-        default: BP_DIAG(8); break;
+        case 8: BP_DIAG(8); break;
+        default: BP_DIAG(kWidePG); break;
     }
 #undef BP_DIAG
     return cudaGetLastError();
