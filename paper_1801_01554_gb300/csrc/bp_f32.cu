@@ -45,6 +45,7 @@ constexpr int kWarps = kThreads / 32;
 constexpr int kTU = 8;            // weight-tile rows (output units)
 constexpr int kTJ = 32;           // weight-tile columns (inputs; the bias is the last input)
 constexpr int kPC = 256;          // patterns per staged chunk of the weight phase
+static_assert(kPC % (kWarps * 4) == 0, "each warp takes whole groups of 4 rows of a chunk");
 constexpr int kChunkFloats = kPC * (kTU + kTJ);
 constexpr int kNBuf = 3;          // chunk buffers in flight
 constexpr int kWidePG = 32;       // patterns per pass of the whole-row-per-lane forward
@@ -777,12 +778,16 @@ __device__ __forceinline__ void issue_chunk(const F32View& v, ChunkPipe& pipe, f
 // (fused == false) or apply the update directly.  One CTA per 8 x 32 tile;
 // the tile's delta and activation blocks stream through shared memory in
 // chunks of kPC patterns, one bulk copy each from the blocked scratch, kNBuf
-// chunks in flight.  Warp w owns a 4 x 4 block of the tile (units 4 (w / 8) ..,
-// columns 4 (w % 8) ..) and lane l the patterns l, l + 32, ... of every chunk,
-// so each pattern feeds 16 FMAs from two 16-byte loads; the 32 lanes' sums then
-// meet by a butterfly inside the warp.  The blocks' row chunks are stored
-// permuted by pattern (see F32View), which keeps the lanes' reads of 32
-// consecutive rows free of bank conflicts.
+// chunks in flight.  Every warp computes the whole tile over its sixteenth of
+// each chunk's patterns (16 consecutive rows): lane l owns column quad l % 8
+// and pattern lane l / 8, holds all 8 units x its 4 columns (32 sums), and
+// takes rows 4 i + l / 8 of the warp's 16.  A pattern then costs two 16-byte
+// delta loads shared by the 8 lanes of a pattern lane and one 16-byte
+// activation load for 32 FMAs, which keeps the loop off the shared-memory
+// bandwidth limit.  The blocks' row chunks are stored permuted by pattern (see
+// F32View), so the lanes' reads are conflict-free.  The sums meet first across
+// the 4 pattern lanes (butterfly), then across the 16 warps in shared memory
+// in warp order: the result does not depend on timing.
 //
 // Returns false (in every thread) if a chunk copy did not arrive in time: no
 // more copies are then issued, every copy already issued has been drained, no
@@ -791,7 +796,7 @@ __device__ bool weight_phase(const F32View& v, int B, bool fused, bool fold_g, f
                              ChunkPipe& pipe) {
     const int tid = threadIdx.x;
     const int lane = tid & 31, warp = tid >> 5;
-    const int uq = warp >> 3, cq = warp & 7;
+    const int cq = lane & 7, pl = lane >> 3;
     float* wbuf = reinterpret_cast<float*>((reinterpret_cast<uintptr_t>(smem) + 1023) & ~(uintptr_t)1023);
     const int L = v.L;
     const int ntiles = v.tile0[L + 1];
@@ -809,21 +814,22 @@ __device__ bool weight_phase(const F32View& v, int B, bool fused, bool fold_g, f
         const int u0 = tb * kTU, j0 = cb * kTJ;
         // the tile's blocks exist in the scratch layout
         if (!bounds_ok(tb < v.dtb[l] && cb < v.acb[l - 1], v.flags)) return true;
-        // this lane's output (lanes 0..15 of each warp) and its current weight
-        // state, loaded now so that their latency hides behind the chunks
-        const int uu = u0 + uq * 4 + ((lane & 15) >> 2), ii = j0 + cq * 4 + (lane & 3);
-        const bool mine = lane < 16 && uu < n_out && ii <= n_in;
+        // the output of threads 0..255 (unit tid / 32, column tid % 32) and its
+        // current weight state, loaded now so that their latency hides behind
+        // the chunks
+        const int uu = u0 + (tid >> 5), ii = j0 + (tid & 31);
+        const bool mine = tid < kTU * kTJ && uu < n_out && ii <= n_in;
         const long long idx = v.woff[l] + (long long)uu * v.kp[l] + ii;   // ii == n_in: bias
         float v_old = 0.f, g_old = 0.f;
         if (mine) {
             if (fused) v_old = __ldcg(v.V + idx);
             if (!fused || fold_g) g_old = __ldcg(v.G + idx);
         }
-        float acc[16];
+        float acc[32];   // unit u, column q of this lane's quad at u * 4 + q
 #pragma unroll
-        for (int k = 0; k < 16; ++k) acc[k] = 0.f;
-        // the buffers' previous contents (weights, pattern rows, the last tile)
-        // were read through the generic proxy by every thread before this sync
+        for (int k = 0; k < 32; ++k) acc[k] = 0.f;
+        // the buffers' previous contents (weights, pattern rows, the last tile's
+        // sums) were read through the generic proxy by every thread before this sync
         __syncthreads();
         if (tid == 0) {
             asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
@@ -844,15 +850,17 @@ __device__ bool weight_phase(const F32View& v, int B, bool fused, bool fold_g, f
                 for (int e = tid; e < (kPC - pc) * kTJ; e += kThreads) As[pc * kTJ + e] = 0.f;
                 __syncthreads();
             }
-#pragma unroll 4
-            for (int k = 0; k < kPC / 32; ++k) {
-                const int p = k * 32 + lane;
-                const float4 d = *reinterpret_cast<const float4*>(Ds + p * kTU + ((uq ^ ((p >> 2) & 1)) << 2));
+#pragma unroll
+            for (int i = 0; i < kPC / (kWarps * 4); ++i) {
+                const int p = warp * (kPC / kWarps) + 4 * i + pl;   // row of the chunk
+                const int dsw = (p >> 2) & 1;
+                const float4 d0 = *reinterpret_cast<const float4*>(Ds + p * kTU + (dsw << 2));
+                const float4 d1 = *reinterpret_cast<const float4*>(Ds + p * kTU + ((1 ^ dsw) << 2));
                 const float4 a = *reinterpret_cast<const float4*>(As + p * kTJ + ((cq ^ (p & 7)) << 2));
-                const float dv[4] = {d.x, d.y, d.z, d.w};
+                const float dv[8] = {d0.x, d0.y, d0.z, d0.w, d1.x, d1.y, d1.z, d1.w};
                 const float av[4] = {a.x, a.y, a.z, a.w};
 #pragma unroll
-                for (int u = 0; u < 4; ++u)
+                for (int u = 0; u < 8; ++u)
 #pragma unroll
                     for (int q = 0; q < 4; ++q) acc[u * 4 + q] = fmaf(dv[u], av[q], acc[u * 4 + q]);
             }
@@ -875,12 +883,37 @@ __device__ bool weight_phase(const F32View& v, int B, bool fused, bool fold_g, f
                 issue_chunk(v, pipe, wbuf, l, tb, cb, c + kNBuf, min(kPC, B - (c + kNBuf) * kPC));
             }
         }
-        // sum over the warp's 32 pattern lanes (fixed order): afterwards lane s
-        // (s < 16) holds value s = (unit u, column q) = (s / 4, s % 4)
-        reduce_scatter<16>(acc, lane);
-        const float g0 = acc[0] + __shfl_xor_sync(0xffffffffu, acc[0], 16);
-        if (lane < 16) {
-            float g = g0;
+        // sum over the 4 pattern lanes (lane bits 4, 3), halving the values at
+        // each level: afterwards the lane holds values base .. base + 7 (units
+        // base / 4 and base / 4 + 1), base = 16 bit4 + 8 bit3
+#pragma unroll
+        for (int k = 0; k < 16; ++k) {
+            const bool up = (lane & 16) != 0;
+            const float send = up ? acc[k] : acc[k + 16];
+            const float keep = up ? acc[k + 16] : acc[k];
+            acc[k] = keep + __shfl_xor_sync(0xffffffffu, send, 16);
+        }
+#pragma unroll
+        for (int k = 0; k < 8; ++k) {
+            const bool up = (lane & 8) != 0;
+            const float send = up ? acc[k] : acc[k + 8];
+            const float keep = up ? acc[k + 8] : acc[k];
+            acc[k] = keep + __shfl_xor_sync(0xffffffffu, send, 8);
+        }
+        // every warp's sums of the tile to shared memory ([warp][unit * 32 + column]);
+        // the chunk buffers are free now
+        float* red = wbuf;
+        const int ub = ((lane >> 4) & 1) * 4 + ((lane >> 3) & 1) * 2;   // first of this lane's two units
+        __syncthreads();
+        *reinterpret_cast<float4*>(red + warp * (kTU * kTJ) + ub * kTJ + 4 * cq) =
+            make_float4(acc[0], acc[1], acc[2], acc[3]);
+        *reinterpret_cast<float4*>(red + warp * (kTU * kTJ) + (ub + 1) * kTJ + 4 * cq) =
+            make_float4(acc[4], acc[5], acc[6], acc[7]);
+        __syncthreads();
+        if (tid < kTU * kTJ) {
+            float g = 0.f;
+#pragma unroll
+            for (int w = 0; w < kWarps; ++w) g += red[w * (kTU * kTJ) + tid];
             if (mine) {
                 if (!fused) {
                     v.G[idx] = g_old + g;
