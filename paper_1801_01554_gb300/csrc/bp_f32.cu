@@ -233,8 +233,18 @@ __device__ __forceinline__ void mbar_drain(uint64_t* bar, unsigned parity) {
     }
 }
 
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
+template <int N>
+__device__ __forceinline__ void cp_async_wait() { asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory"); }
+__device__ __forceinline__ void cp_async4(float* dst, const float* src) {
+    asm volatile("cp.async.ca.shared.global [%0], [%1], 4;" ::"r"(smem_u32(dst)), "l"(src) : "memory");
+}
+
 // Starts the copy of theta[0, P) into shared memory Ws: one bulk copy on the
-// mbarrier for the 16-byte aligned part (thread 0), plain loads for the tail.
+// mbarrier for the 16-byte aligned part (thread 0), and 4-byte cp.async copies
+// for the tail of at most 3 floats by the last threads (no thread stalls on a
+// load here; the tail belongs to the issuing thread's next cp.async group,
+// which stage_weights_wait waits for).
 __device__ void stage_weights_issue(const float* theta, long long P, float* Ws, uint64_t* bar) {
     const long long P16 = P & ~3LL;
     if (threadIdx.x == 0 && P16 > 0) {
@@ -250,32 +260,41 @@ __device__ void stage_weights_issue(const float* theta, long long P, float* Ws, 
             "l"(theta), "r"(bytes), "r"(smem_u32(bar))
             : "memory");
     }
-    for (long long k = P16 + threadIdx.x; k < P; k += kThreads) Ws[k] = __ldcg(theta + k);
+    const long long k = P16 + (kThreads - 1 - (int)threadIdx.x);
+    if (k < P) cp_async4(Ws + k, theta + k);
 }
 
 // Bounded wait for a copy started by stage_weights_issue (every thread; the
-// tail written by plain stores needs a CTA barrier after this).  Returns false
-// in a thread whose wait ran out; callers make that CTA-uniform with
+// tail needs a CTA barrier after this).  The thread's cp.async groups are
+// waited for too (the tail's, and any rows issued since).  Returns false in a
+// thread whose wait ran out; callers make that CTA-uniform with
 // __syncthreads_or and then call stage_weights_drain before returning.
+// A copy in flight: its mbarrier (none if bar is null), the parity of the
+// phase it completes, and its length.  Passed by value, so that nothing of it
+// lives in local memory.
 struct WeightCopy {
     uint64_t* bar;
-    unsigned* phase;
+    unsigned parity;
     long long P;
 };
 __device__ __forceinline__ bool stage_weights_wait(const WeightCopy& w, int* flags) {
     bool ok = true;
-    if ((w.P & ~3LL) > 0) {
-        ok = mbar_wait(w.bar, *w.phase, flags);
-        *w.phase ^= 1u;
-    }
+    if (w.bar != nullptr && (w.P & ~3LL) > 0) ok = mbar_wait(w.bar, w.parity, flags);
+    cp_async_commit();
+    cp_async_wait<0>();
     return ok;
+}
+
+// The mbarrier phase parity after a copy started by stage_weights_issue.
+__device__ __forceinline__ unsigned after_copy(unsigned parity, long long P) {
+    return (P & ~3LL) > 0 ? parity ^ 1u : parity;
 }
 
 // After a weight copy whose wait ran out in some thread: thread 0 waits for
 // that copy again (bounded) so that no bulk write is still landing when the CTA
 // returns.  Every thread calls it.
 __device__ void stage_weights_drain(const WeightCopy& w) {
-    if (threadIdx.x == 0 && (w.P & ~3LL) > 0) mbar_drain(w.bar, *w.phase ^ 1u);
+    if (threadIdx.x == 0 && w.bar != nullptr && (w.P & ~3LL) > 0) mbar_drain(w.bar, w.parity);
     __syncthreads();
 }
 
@@ -285,7 +304,8 @@ __device__ void stage_weights_drain(const WeightCopy& w) {
 __device__ bool stage_weights(const float* theta, long long P, float* Ws, uint64_t* bar,
                               unsigned& phase, int* flags) {
     stage_weights_issue(theta, P, Ws, bar);
-    const WeightCopy wc{bar, &phase, P};
+    const WeightCopy wc{bar, phase, P};
+    phase = after_copy(phase, P);
     if (__syncthreads_or(!stage_weights_wait(wc, flags))) {
         stage_weights_drain(wc);
         return false;
@@ -294,12 +314,6 @@ __device__ bool stage_weights(const float* theta, long long P, float* Ws, uint64
 }
 
 // ------------------------------------------------------------ pattern phase
-__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
-template <int N>
-__device__ __forceinline__ void cp_async_wait() { asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory"); }
-__device__ __forceinline__ void cp_async4(float* dst, const float* src) {
-    asm volatile("cp.async.ca.shared.global [%0], [%1], 4;" ::"r"(smem_u32(dst)), "l"(src) : "memory");
-}
 
 // Shared memory: the weights (WS) at the bottom, the pattern buffers above
 // them; the weight phase reuses the bottom kGradFloats floats for its tiles.
@@ -480,6 +494,64 @@ __device__ void forward_layer_lanes(const float* W, int kp, int n_out, const flo
     }
 }
 
+// Forward through one layer for groups of 32 patterns, register-blocked: lane
+// l holds patterns l % 16 and l % 16 + 16 of its warp's group and units
+// j0 + 4 (l / 16) .. + 3 of the warp's 8, so every activation float4 feeds 16
+// FMAs and every weight float4 8.  A warp's loads per float4 step are two
+// activation reads of 16 rows each and four weight reads of 2 rows each (4
+// rows apart), for 32 FMAs per lane.  With kp / 4 odd (f32_plan checks it) the
+// 16 rows fall on 8 distinct 16-byte bank groups twice (two wavefronts, the
+// minimum for 256 bytes) and the two weight rows, kp float4 apart, on
+// different bank groups (one wavefront each).
+template <int PG>
+__device__ void forward_layer_blocked(const float* W, int kp, int n_out, const float* s_in, float* s_out,
+                                      int kp_out, bool table) {
+    static_assert(PG % 32 == 0, "whole warps of patterns");
+    constexpr int kGroups = PG / 32;
+    constexpr int kWarpsPerGroup = kWarps / kGroups;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int p0 = (warp / kWarpsPerGroup) * 32 + (lane & 15), wi = warp % kWarpsPerGroup;
+    const int K4 = kp >> 2;
+    const float* a0 = s_in + p0 * kp;
+    const float* a1 = a0 + 16 * kp;
+    for (int jb = wi * 8; jb < n_out; jb += kWarpsPerGroup * 8) {
+        const int j0 = jb + 4 * (lane >> 4);
+        const float* w0 = W + min(j0, n_out - 1) * kp;   // rows past the layer repeat its last row
+        const float* w1 = W + min(j0 + 1, n_out - 1) * kp;
+        const float* w2 = W + min(j0 + 2, n_out - 1) * kp;
+        const float* w3 = W + min(j0 + 3, n_out - 1) * kp;
+        float c0[4] = {0.f, 0.f, 0.f, 0.f}, c1[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll 2
+        for (int k = 0; k < K4; ++k) {
+            const float4 x0 = ld4(a0 + 4 * k), x1 = ld4(a1 + 4 * k);
+            const float4 w[4] = {ld4(w0 + 4 * k), ld4(w1 + 4 * k), ld4(w2 + 4 * k), ld4(w3 + 4 * k)};
+#pragma unroll
+            for (int u = 0; u < 4; ++u) {
+                float t0 = c0[u], t1 = c1[u];
+                t0 = fmaf(w[u].x, x0.x, t0);
+                t1 = fmaf(w[u].x, x1.x, t1);
+                t0 = fmaf(w[u].y, x0.y, t0);
+                t1 = fmaf(w[u].y, x1.y, t1);
+                t0 = fmaf(w[u].z, x0.z, t0);
+                t1 = fmaf(w[u].z, x1.z, t1);
+                t0 = fmaf(w[u].w, x0.w, t0);
+                t1 = fmaf(w[u].w, x1.w, t1);
+                c0[u] = t0;
+                c1[u] = t1;
+            }
+        }
+        float* o0 = s_out + p0 * kp_out + j0;
+        float* o1 = o0 + 16 * kp_out;
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+            if (j0 + u < n_out) {
+                o0[u] = table ? sigmoid_tab(c0[u]) : sigmoid_f(c0[u]);
+                o1[u] = table ? sigmoid_tab(c1[u]) : sigmoid_f(c1[u]);
+            }
+        }
+    }
+}
+
 // Forward through one layer for PG patterns held in shared memory: the
 // lane-group form below for small groups, whole rows per lane from 32 up.
 template <int PG>
@@ -487,7 +559,7 @@ __device__ __forceinline__ void forward_any(const float* W, int kp, int n_out, c
                                             int kp_out, bool table) {
     if constexpr (PG >= 32) {
         if (n_out >= 4 * kWarps / (PG / 32))
-            forward_layer_lanes<PG, 8>(W, kp, n_out, s_in, s_out, kp_out, table);
+            forward_layer_blocked<PG>(W, kp, n_out, s_in, s_out, kp_out, table);
         else
             forward_layer_lanes<PG, 2>(W, kp, n_out, s_in, s_out, kp_out, table);
     } else {
@@ -602,22 +674,26 @@ __device__ __forceinline__ void rows_to_scratch(const F32View& v, int l, const f
 //   do_fwd: forward pass from X (else the activations are reloaded from scratch)
 //   do_bwd: deltas against T, written to scratch
 //   Y: if not null, the outputs are copied there ([B, n_L] packed)
-// Returns this CTA's summed squared error (valid in thread 0).
-//   wc: if not null, a weight copy into shared memory is still in flight; it
-//       is waited for after the first rows have been issued, so that the two
-//       loads overlap
+// Returns this CTA's summed squared error (valid in thread 0) and whether the
+// weight copy arrived.
+//   wc: if wc.bar is not null, a weight copy into shared memory is still in
+//       flight; it is waited for after the first rows have been issued, so
+//       that the two loads overlap
 //   to_scratch: write the activation and delta rows to scratch (A, D)
 //   rows_issued: the first pass's rows were already issued (load_rows)
 //   whole: this CTA takes all B patterns (diagnostic mode) instead of its share
-//   copy_ok: with wc, set false (in every thread) if the weight copy timed out;
-//       it has then been drained and the phase did nothing, so the caller returns
+// ok is false (in every thread) if the weight copy timed out: it has then been
+// drained and the phase did nothing, so the caller returns.
+struct PhaseResult {
+    float sse;
+    bool ok;
+};
 template <int PG>
-__device__ float pattern_phase(const F32View& v, const PatLayout& q, const float* Wb,
-                               const float* __restrict__ X, const float* __restrict__ T, int B,
-                               bool do_fwd, bool do_bwd, float* __restrict__ Y, float* smem,
-                               const WeightCopy* wc = nullptr, bool to_scratch = true,
-                               bool rows_issued = false, bool whole = false,
-                               bool* copy_ok = nullptr) {
+__device__ PhaseResult pattern_phase(const F32View& v, const PatLayout& q, const float* Wb,
+                                     const float* __restrict__ X, const float* __restrict__ T, int B,
+                                     bool do_fwd, bool do_bwd, float* __restrict__ Y, float* smem,
+                                     WeightCopy wc = WeightCopy{nullptr, 0u, 0}, bool to_scratch = true,
+                                     bool rows_issued = false, bool whole = false) {
     constexpr int TP = kThreads / PG;
     const int L = v.L;
     const int tid = threadIdx.x;
@@ -626,16 +702,14 @@ __device__ float pattern_phase(const F32View& v, const PatLayout& q, const float
     float sse = 0.f;
     const int q_lo = whole ? 0 : (int)((long long)B * blockIdx.x / gridDim.x);
     const int q_hi = whole ? B : (int)((long long)B * (blockIdx.x + 1) / gridDim.x);
-    if (copy_ok != nullptr) *copy_ok = true;
     if (!bounds_ok((size_t)(smem - pattern_smem_base()) + q.total <= dyn_smem_floats() &&
                        ((!to_scratch && do_fwd) || B <= v.cap),
                    v.flags)) {
-        if (wc != nullptr && __syncthreads_or(!stage_weights_wait(*wc, v.flags))) {
-            stage_weights_drain(*wc);
-            if (copy_ok != nullptr) *copy_ok = false;
-            return 0.f;
+        if (wc.bar != nullptr && __syncthreads_or(!stage_weights_wait(wc, v.flags))) {
+            stage_weights_drain(wc);
+            return PhaseResult{0.f, false};
         }
-        return block_sum(0.f);
+        return PhaseResult{block_sum(0.f), true};
     }
     for (int p0 = q_lo; p0 < q_hi; p0 += PG) {
         const int np = min(PG, q_hi - p0);
@@ -651,17 +725,16 @@ __device__ float pattern_phase(const F32View& v, const PatLayout& q, const float
             }
         }
         bool w_ok = true;
-        const WeightCopy* waited = wc;
-        if (wc != nullptr) {
-            w_ok = stage_weights_wait(*wc, v.flags);
-            wc = nullptr;
+        const WeightCopy waited = wc;
+        if (wc.bar != nullptr) {
+            w_ok = stage_weights_wait(wc, v.flags);
+            wc.bar = nullptr;
         }
         cp_async_wait<0>();
         if (__syncthreads_or(!w_ok)) {
             // the weight copy did not arrive in time: let it land, do nothing more
-            stage_weights_drain(*waited);
-            if (copy_ok != nullptr) *copy_ok = false;
-            return 0.f;
+            stage_weights_drain(waited);
+            return PhaseResult{0.f, false};
         }
         if (do_fwd) {
             // the input rows go to scratch first, so that their stores drain during the forward pass
@@ -712,14 +785,13 @@ __device__ float pattern_phase(const F32View& v, const PatLayout& q, const float
         }
         __syncthreads();
     }
-    if (wc != nullptr && __syncthreads_or(!stage_weights_wait(*wc, v.flags))) {   // no patterns here
-        stage_weights_drain(*wc);
-        if (copy_ok != nullptr) *copy_ok = false;
-        return 0.f;
+    if (wc.bar != nullptr && __syncthreads_or(!stage_weights_wait(wc, v.flags))) {   // no patterns here
+        stage_weights_drain(wc);
+        return PhaseResult{0.f, false};
     }
     // the weight phase reads the activation and delta rows through TMA
     asm volatile("fence.proxy.async.global;" ::: "memory");
-    return block_sum(sse);
+    return PhaseResult{block_sum(sse), true};
 }
 
 // ------------------------------------------------------------ weight phase
@@ -773,6 +845,39 @@ __device__ __forceinline__ void issue_chunk(const F32View& v, ChunkPipe& pipe, f
     bulk_load(buf + kPC * kTJ, v.D + v.doff[l] + (long long)tb * v.cap * kTU + p0 * kTU, dbytes, pipe.bar + b);
 }
 
+// Tile t of the weight phase: its layer l, block row tb (units 8 tb ..) and
+// block column cb (inputs 32 cb ..).
+struct Tile {
+    int l, tb, cb;
+};
+__device__ __forceinline__ Tile tile_at(const F32View& v, int t) {
+    int l = 1;
+    while (t >= v.tile0[l + 1]) ++l;
+    const int lt = t - v.tile0[l];
+    const int tb = lt / v.tcols[l];
+    return Tile{l, tb, lt - tb * v.tcols[l]};
+}
+
+// The weight phase's chunk buffers: the bottom of shared memory, aligned to 1 KB.
+__device__ __forceinline__ float* chunk_buffers(float* smem) {
+    return reinterpret_cast<float*>((reinterpret_cast<uintptr_t>(smem) + 1023) & ~(uintptr_t)1023);
+}
+__device__ __forceinline__ bool chunk_buffers_fit(const F32View& v, int B, const float* wbuf) {
+    return (size_t)(wbuf - pattern_smem_base()) + kNBuf * kChunkFloats <= dyn_smem_floats() && B <= v.cap;
+}
+
+// Thread 0: the first kNBuf chunk copies of a tile.  The proxy fences order
+// the buffers' earlier generic-proxy reads and the scratch rows' generic-proxy
+// writes before the bulk copies.
+__device__ __forceinline__ void issue_tile_start(const F32View& v, ChunkPipe& pipe, float* wbuf,
+                                                 const Tile& tl, int B) {
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+    asm volatile("fence.proxy.async.global;" ::: "memory");
+    const int nchunks = (B + kPC - 1) / kPC;
+    for (int c = 0; c < nchunks && c < kNBuf; ++c)
+        issue_chunk(v, pipe, wbuf, tl.l, tl.tb, tl.cb, c, min(kPC, B - c * kPC));
+}
+
 // Pooled change of every weight (and bias: the last input column is the true
 // unit's 1) over the B patterns of the group, then either accumulate into G
 // (fused == false) or apply the update directly.  One CTA per 8 x 32 tile;
@@ -797,23 +902,22 @@ __device__ bool weight_phase(const F32View& v, int B, bool fused, bool fold_g, f
     const int tid = threadIdx.x;
     const int lane = tid & 31, warp = tid >> 5;
     const int cq = lane & 7, pl = lane >> 3;
-    float* wbuf = reinterpret_cast<float*>((reinterpret_cast<uintptr_t>(smem) + 1023) & ~(uintptr_t)1023);
+    float* wbuf = chunk_buffers(smem);
     const int L = v.L;
     const int ntiles = v.tile0[L + 1];
     const int nchunks = (B + kPC - 1) / kPC;
-    if (!bounds_ok((size_t)(wbuf - pattern_smem_base()) + kNBuf * kChunkFloats <= dyn_smem_floats() &&
-                       B <= v.cap,
-                   v.flags))
-        return true;
+    if (!bounds_ok(chunk_buffers_fit(v, B, wbuf), v.flags)) return true;
     for (int t = blockIdx.x; t < ntiles; t += gridDim.x) {
-        int l = 1;
-        while (t >= v.tile0[l + 1]) ++l;
-        const int lt = t - v.tile0[l];
-        const int tb = lt / v.tcols[l], cb = lt - tb * v.tcols[l];
+        const Tile tl = tile_at(v, t);
+        const int l = tl.l, tb = tl.tb, cb = tl.cb;
         const int n_in = v.n[l - 1], n_out = v.n[l];
         const int u0 = tb * kTU, j0 = cb * kTJ;
         // the tile's blocks exist in the scratch layout
         if (!bounds_ok(tb < v.dtb[l] && cb < v.acb[l - 1], v.flags)) return true;
+        // the buffers' previous contents (weights, pattern rows, the last tile's
+        // sums) were read through the generic proxy by every thread before this sync
+        __syncthreads();
+        if (tid == 0) issue_tile_start(v, pipe, wbuf, tl, B);
         // the output of threads 0..255 (unit tid / 32, column tid % 32) and its
         // current weight state, loaded now so that their latency hides behind
         // the chunks
@@ -828,15 +932,6 @@ __device__ bool weight_phase(const F32View& v, int B, bool fused, bool fold_g, f
         float acc[32];   // unit u, column q of this lane's quad at u * 4 + q
 #pragma unroll
         for (int k = 0; k < 32; ++k) acc[k] = 0.f;
-        // the buffers' previous contents (weights, pattern rows, the last tile's
-        // sums) were read through the generic proxy by every thread before this sync
-        __syncthreads();
-        if (tid == 0) {
-            asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-            asm volatile("fence.proxy.async.global;" ::: "memory");
-            for (int c = 0; c < nchunks && c < kNBuf; ++c)
-                issue_chunk(v, pipe, wbuf, l, tb, cb, c, min(kPC, B - c * kPC));
-        }
         for (int c = 0; c < nchunks; ++c) {
             const int b = c % kNBuf;
             const bool got = mbar_wait(pipe.bar + b, (pipe.parity >> b) & 1u, v.flags);
@@ -965,7 +1060,7 @@ __device__ void reduce_sse(const F32View& v, int nparts, float* sse_out) {
 // WS: the weights are copied into shared memory (else read from global memory).
 template <int PG, bool WS>
 __global__ void __launch_bounds__(kThreads, 1)
-    k_forward(const __grid_constant__ F32View v, const PatLayout q, const float* X, int B, float* Y) {
+    k_forward(const __grid_constant__ F32View v, const __grid_constant__ PatLayout q, const float* X, int B, float* Y) {
     extern __shared__ __align__(128) float smem[];
     __shared__ __align__(8) uint64_t s_bar;
     unsigned phase = 0;
@@ -983,7 +1078,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 
 template <int PG, bool WS>
 __global__ void __launch_bounds__(kThreads, 1)
-    k_deltas(const __grid_constant__ F32View v, const PatLayout q, const float* T, int B) {
+    k_deltas(const __grid_constant__ F32View v, const __grid_constant__ PatLayout q, const float* T, int B) {
     extern __shared__ __align__(128) float smem[];
     __shared__ __align__(8) uint64_t s_bar;
     unsigned phase = 0;
@@ -992,9 +1087,9 @@ __global__ void __launch_bounds__(kThreads, 1)
         mbar_init1(&s_bar);
         if (!bounds_ok((unsigned)v.wsm <= dyn_smem_floats(), v.flags)) return;
         if (!stage_weights(v.theta, v.P, smem, &s_bar, phase, v.flags)) return;
-        e = pattern_phase<PG>(v, q, smem, nullptr, T, B, false, true, nullptr, pattern_base<true>(v, smem));
+        e = pattern_phase<PG>(v, q, smem, nullptr, T, B, false, true, nullptr, pattern_base<true>(v, smem)).sse;
     } else {
-        e = pattern_phase<PG>(v, q, v.theta, nullptr, T, B, false, true, nullptr, pattern_base<false>(v, smem));
+        e = pattern_phase<PG>(v, q, v.theta, nullptr, T, B, false, true, nullptr, pattern_base<false>(v, smem)).sse;
     }
     if (threadIdx.x == 0) v.sse_part[blockIdx.x] = e;
 }
@@ -1004,7 +1099,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 // reports its summed squared error and the SM it ran on.
 template <int PG, bool WS>
 __global__ void __launch_bounds__(kThreads, 1)
-    k_diagnose(const __grid_constant__ F32View v, const PatLayout q, const float* X, const float* T,
+    k_diagnose(const __grid_constant__ F32View v, const __grid_constant__ PatLayout q, const float* X, const float* T,
                int B, float* sse_out, int* sm_out) {
     extern __shared__ __align__(128) float smem[];
     __shared__ __align__(8) uint64_t s_bar;
@@ -1016,10 +1111,10 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (WS) {
         if (!stage_weights(v.theta, v.P, smem, &s_bar, phase, v.flags)) return;
         e = pattern_phase<PG>(v, q, smem, X, T, B, true, true, nullptr, pattern_base<true>(v, smem),
-                              nullptr, false, false, true);
+                              WeightCopy{nullptr, 0u, 0}, false, false, true).sse;
     } else {
         e = pattern_phase<PG>(v, q, v.theta, X, T, B, true, true, nullptr, pattern_base<false>(v, smem),
-                              nullptr, false, false, true);
+                              WeightCopy{nullptr, 0u, 0}, false, false, true).sse;
     }
     if (threadIdx.x == 0) {
         unsigned sm;
@@ -1051,7 +1146,7 @@ __global__ void __launch_bounds__(256) k_update(const __grid_constant__ F32View 
 
 template <int PG, bool WS>
 __global__ void __launch_bounds__(kThreads, 1)
-    k_train(const __grid_constant__ F32View v, const PatLayout q, const float* X, const float* T,
+    k_train(const __grid_constant__ F32View v, const __grid_constant__ PatLayout q, const float* X, const float* T,
             int n_patterns, int minibatch, int n_steps, float* sse_out, int fold_g) {
     extern __shared__ __align__(128) float smem[];
     __shared__ __align__(8) uint64_t s_bar;
@@ -1078,13 +1173,13 @@ __global__ void __launch_bounds__(kThreads, 1)
         float e;
         if (WS) {
             stage_weights_issue(v.theta, v.P, smem, &s_bar);
-            const WeightCopy wc{&s_bar, &phase, v.P};
-            bool copy_ok = true;
-            e = pattern_phase<PG>(v, q, smem, Xs, Ts, B, true, true, nullptr, pat, &wc, true, false,
-                                  false, &copy_ok);
-            if (!copy_ok) return;   // the copy was drained; the error is latched
+            const WeightCopy wc{&s_bar, phase, v.P};
+            phase = after_copy(phase, v.P);
+            const PhaseResult r = pattern_phase<PG>(v, q, smem, Xs, Ts, B, true, true, nullptr, pat, wc);
+            if (!r.ok) return;   // the copy was drained; the error is latched
+            e = r.sse;
         } else {
-            e = pattern_phase<PG>(v, q, v.theta, Xs, Ts, B, true, true, nullptr, pat);
+            e = pattern_phase<PG>(v, q, v.theta, Xs, Ts, B, true, true, nullptr, pat).sse;
         }
         if (threadIdx.x == 0) v.sse_part[blockIdx.x] = e;
         if (!grid_barrier(v.bar, target += gridDim.x, v.flags, wait_limit_ns(v))) return;
@@ -1116,6 +1211,8 @@ struct SmallPlan {
 
 // GUARD: the fault guard is on (a separate instantiation, so that the update
 // loop carries no test when it is off).
+// (The pattern layout and plan are by-value parameters here: as grid constants
+// they cost this kernel register spills at 16 update slots.)
 template <int PG, int NV4, bool GUARD>
 __global__ void __launch_bounds__(kThreads, 1)
     k_train_small(const __grid_constant__ F32View v, const PatLayout q, const SmallPlan sp,
@@ -1153,7 +1250,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int B = (int)min((long long)minibatch, (long long)n_patterns - p0);
         float* ps = pat[s & 1];
         const float e = pattern_phase<PG>(v, q, smem, X + p0 * n0, T + p0 * nL, B, true, true, nullptr,
-                                          ps, nullptr, false, true);
+                                          ps, WeightCopy{nullptr, 0u, 0}, false, true).sse;
         if (tid == 0) {
             if (sse_out != nullptr) sse_out[s] = e;
             if (!isfinite(e)) atomicOr(v.flags, kFlagNonfinite);

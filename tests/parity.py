@@ -17,6 +17,9 @@ kappa_l = max(|D|_l^T |A_{l-1}|) / max|G_l| is 1 when nothing cancels and
 grows when the terms of the sums cancel (deep nets whose first-layer changes
 are much smaller than their terms).  The float32 bar of 1e-5 is applied to the
 sum's magnitude: the allowed normwise error of layer l is 1e-5 * max(1, kappa_l).
+kappa uses the same floor for max|G_l| as normwise() does for the reference's
+size, so that for a change that is exactly zero the bar is the absolute bound
+1e-5 * max(|D|_l^T |A_{l-1}|).
 """
 import numpy as np
 
@@ -57,8 +60,8 @@ def kappa(sizes, theta, X, T, squash="logistic"):
         Gm = mag[l].T @ np.abs(As[l])
         g = Ds[l].sum(axis=0)
         gm = mag[l].sum(axis=0)
-        out.append(max(1.0, float(Gm.max() / max(np.abs(G).max(), 1e-300))))
-        out.append(max(1.0, float(gm.max() / max(np.abs(g).max(), 1e-300))))
+        out.append(max(1.0, float(Gm.max() / max(np.abs(G).max(), 1e-30))))
+        out.append(max(1.0, float(gm.max() / max(np.abs(g).max(), 1e-30))))
     return out
 
 

@@ -50,12 +50,14 @@ def check_state(sizes, theta0, W, V, st, kap, what, n_upd=1):
     """End state of a run of n_upd updates against the oracle's: W - W0 and V
     per layer.  W - W0 carries the rounding of the stored float32 weights after
     every update (half an ulp of |W| each), which sets its floor when the
-    change is small next to the weights."""
+    change is small next to the weights.  The floor of the reference's size is
+    the one normwise() divides by, so that a part whose reference change is
+    exactly zero gets the absolute bar n_upd * u * max|W| (in float64)."""
     kap = kap or [1.0] * (2 * (len(sizes) - 1))
     floor = []
     for k, (lab, sl) in zip(kap, layer_parts(sizes)):
-        dref = max(np.max(np.abs(st.theta[sl] - theta0[sl])), 1e-300)
-        floor.append(k + n_upd * U32 * np.max(np.abs(st.theta[sl])) / (TOL * dref))
+        dref = max(float(np.max(np.abs(st.theta[sl] - theta0[sl]))), 1e-30)
+        floor.append(k + n_upd * U32 * float(np.max(np.abs(st.theta[sl]))) / (TOL * dref))
     e = assert_layers(sizes, W - theta0, st.theta - theta0, TOL, floor, what + " W-W0")
     assert_layers(sizes, V, st.V, TOL, kap, what + " V")
     return e
@@ -65,11 +67,14 @@ def change_bar(sizes, kap, V_k, dv_ref):
     """Bar factors for a step's change lr*G read back as V_k - m*V_prev: the
     stored float32 V_k rounds it (two roundings of |V_k|), which dominates when
     the momentum term is much larger than the change (a net whose changes have
-    died out in saturation)."""
+    died out in saturation).  A part whose reference change is exactly zero (a
+    saturated layer) gets the absolute bar 2 u max|V_k|: the floor of the
+    reference's size is the one normwise() divides by, and the arithmetic is
+    float64 (a float32 quotient would round the bar to infinity)."""
     out = []
     for k, (lab, sl) in zip(kap, layer_parts(sizes)):
-        dref = max(np.max(np.abs(dv_ref[sl])), 1e-300)
-        out.append(k + 2 * U32 * np.max(np.abs(V_k[sl])) / (TOL * dref))
+        dref = max(float(np.max(np.abs(dv_ref[sl]))), 1e-30)
+        out.append(k + 2 * U32 * float(np.max(np.abs(V_k[sl]))) / (TOL * dref))
     return out
 
 
