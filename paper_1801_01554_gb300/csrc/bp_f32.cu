@@ -18,7 +18,7 @@
 //   weight phase (Section 5's "bundle" of weights processed over the whole
 //     group of cases): one CTA per 8 x 32 tile of [W_l | b_l] streams the
 //     group's deltas and activations through shared memory, two contiguous
-//     bulk copies per chunk of 256 patterns,
+//     bulk copies per chunk of 512 patterns,
 //     sums delta[p,j] a[p,i] over all patterns with 4 x 4 register blocks per
 //     lane and a warp butterfly (Sections 3, 4.1), then either accumulates into
 //     G (bp_backward) or applies the momentum update of Section 6.2.1 at once
@@ -44,10 +44,13 @@ constexpr int kThreads = 512;
 constexpr int kWarps = kThreads / 32;
 constexpr int kTU = 8;            // weight-tile rows (output units)
 constexpr int kTJ = 32;           // weight-tile columns (inputs; the bias is the last input)
-constexpr int kPC = 256;          // patterns per staged chunk of the weight phase
+constexpr int kPC = 512;          // patterns per staged chunk of the weight phase
 static_assert(kPC % (kWarps * 4) == 0, "each warp takes whole groups of 4 rows of a chunk");
 constexpr int kChunkFloats = kPC * (kTU + kTJ);
-constexpr int kNBuf = 3;          // chunk buffers in flight
+constexpr int kWarpRows = kPC / kWarps;   // rows of a chunk per warp
+// chunk buffers in flight: the CTA syncs once per chunk, so the chunk is as
+// large as two buffers allow (256 x 3 and 128 x 6 measured slower)
+constexpr int kNBuf = 2;
 constexpr int kWidePG = 32;       // patterns per pass of the whole-row-per-lane forward
 // weight-phase buffers (each chunk: the [kPC][kTJ] activation block, 128-byte
 // swizzled, then the [kPC][kTU] delta block), plus room to align them to 1 KB
@@ -884,9 +887,9 @@ __device__ __forceinline__ void issue_tile_start(const F32View& v, ChunkPipe& pi
 // the tile's delta and activation blocks stream through shared memory in
 // chunks of kPC patterns, one bulk copy each from the blocked scratch, kNBuf
 // chunks in flight.  Every warp computes the whole tile over its sixteenth of
-// each chunk's patterns (16 consecutive rows): lane l owns column quad l % 8
-// and pattern lane l / 8, holds all 8 units x its 4 columns (32 sums), and
-// takes rows 4 i + l / 8 of the warp's 16.  A pattern then costs two 16-byte
+// each chunk's patterns (kPC / 16 consecutive rows): lane l owns column quad
+// l % 8 and pattern lane l / 8, holds all 8 units x its 4 columns (32 sums),
+// and takes rows 4 i + l / 8 of the warp's share.  A pattern then costs two 16-byte
 // delta loads shared by the 8 lanes of a pattern lane and one 16-byte
 // activation load for 32 FMAs, which keeps the loop off the shared-memory
 // bandwidth limit.  The blocks' row chunks are stored permuted by pattern (see
@@ -940,24 +943,29 @@ __device__ bool weight_phase(const F32View& v, int B, bool fused, bool fold_g, f
             float* Ds = As + kPC * kTJ;
             const int pc = B - c * kPC;
             if (pc < kPC) {
-                // rows past the group may hold stale scratch rows: clear them
-                for (int e = tid; e < (kPC - pc) * kTU; e += kThreads) Ds[pc * kTU + e] = 0.f;
-                for (int e = tid; e < (kPC - pc) * kTJ; e += kThreads) As[pc * kTJ + e] = 0.f;
+                // rows past the group may hold stale scratch rows: clear those
+                // in the share of the last warp with live rows (the warps after
+                // it skip the chunk)
+                const int pend = min(kPC, (pc + kWarpRows - 1) / kWarpRows * kWarpRows);
+                for (int e = tid; e < (pend - pc) * kTU; e += kThreads) Ds[pc * kTU + e] = 0.f;
+                for (int e = tid; e < (pend - pc) * kTJ; e += kThreads) As[pc * kTJ + e] = 0.f;
                 __syncthreads();
             }
+            if (warp * kWarpRows < pc) {   // warp-uniform: the warp has live rows
 #pragma unroll
-            for (int i = 0; i < kPC / (kWarps * 4); ++i) {
-                const int p = warp * (kPC / kWarps) + 4 * i + pl;   // row of the chunk
-                const int dsw = (p >> 2) & 1;
-                const float4 d0 = *reinterpret_cast<const float4*>(Ds + p * kTU + (dsw << 2));
-                const float4 d1 = *reinterpret_cast<const float4*>(Ds + p * kTU + ((1 ^ dsw) << 2));
-                const float4 a = *reinterpret_cast<const float4*>(As + p * kTJ + ((cq ^ (p & 7)) << 2));
-                const float dv[8] = {d0.x, d0.y, d0.z, d0.w, d1.x, d1.y, d1.z, d1.w};
-                const float av[4] = {a.x, a.y, a.z, a.w};
+                for (int i = 0; i < kWarpRows / 4; ++i) {
+                    const int p = warp * kWarpRows + 4 * i + pl;   // row of the chunk
+                    const int dsw = (p >> 2) & 1;
+                    const float4 d0 = *reinterpret_cast<const float4*>(Ds + p * kTU + (dsw << 2));
+                    const float4 d1 = *reinterpret_cast<const float4*>(Ds + p * kTU + ((1 ^ dsw) << 2));
+                    const float4 a = *reinterpret_cast<const float4*>(As + p * kTJ + ((cq ^ (p & 7)) << 2));
+                    const float dv[8] = {d0.x, d0.y, d0.z, d0.w, d1.x, d1.y, d1.z, d1.w};
+                    const float av[4] = {a.x, a.y, a.z, a.w};
 #pragma unroll
-                for (int u = 0; u < 8; ++u)
+                    for (int u = 0; u < 8; ++u)
 #pragma unroll
-                    for (int q = 0; q < 4; ++q) acc[u * 4 + q] = fmaf(dv[u], av[q], acc[u * 4 + q]);
+                        for (int q = 0; q < 4; ++q) acc[u * 4 + q] = fmaf(dv[u], av[q], acc[u * 4 + q]);
+                }
             }
             if (__syncthreads_or(!got)) {
                 // a chunk did not arrive in time: issue nothing more and let
