@@ -66,6 +66,7 @@ struct bp_net {
     float* A = nullptr;
     float* D = nullptr;
     float* sse_part = nullptr;
+    float* wpart = nullptr;
     unsigned* bar = nullptr;
     int* flags = nullptr;
     F32View view{};
@@ -97,6 +98,7 @@ void free_all(bp_net* net) {
     cudaFree(net->A);
     cudaFree(net->D);
     cudaFree(net->sse_part);
+    cudaFree(net->wpart);
     cudaFree(net->bar);
     cudaFree(net->flags);
     cudaFree(net->stage_X);
@@ -217,6 +219,7 @@ bp_status bp_create(const int* sizes, int n_layers, float lr, float momentum, in
         e = cudaMalloc(&net->A, v.a_floats * sizeof(float));
         if (e == cudaSuccess) e = cudaMalloc(&net->D, v.d_floats * sizeof(float));
         if (e == cudaSuccess) e = cudaMalloc(&net->sse_part, (size_t)net->num_sms * 4 * sizeof(float));
+        if (e == cudaSuccess) e = cudaMalloc(&net->wpart, (size_t)net->num_sms * 2 * 256 * sizeof(float));
         if (e == cudaSuccess) e = cudaMalloc(&net->bar, (size_t)bp::kBarWords * sizeof(unsigned));
         if (e == cudaSuccess) e = cudaMalloc(&net->flags, 4 * sizeof(int));
         if (e != cudaSuccess) return bail(cuda_fail(e, "cudaMalloc(scratch)"));
@@ -231,6 +234,7 @@ bp_status bp_create(const int* sizes, int n_layers, float lr, float momentum, in
         v.A = net->A;
         v.D = net->D;
         v.sse_part = net->sse_part;
+        v.wpart = net->wpart;
         v.bar = net->bar;
         v.flags = net->flags;
         v.faults = reinterpret_cast<unsigned*>(net->flags + 1);

@@ -869,16 +869,50 @@ __device__ __forceinline__ bool chunk_buffers_fit(const F32View& v, int B, const
     return (size_t)(wbuf - pattern_smem_base()) + kNBuf * kChunkFloats <= dyn_smem_floats() && B <= v.cap;
 }
 
-// Thread 0: the first kNBuf chunk copies of a tile.  The proxy fences order
-// the buffers' earlier generic-proxy reads and the scratch rows' generic-proxy
-// writes before the bulk copies.
+// Thread 0: the first kNBuf chunk copies of chunks [c0, c1) of a tile.  The
+// proxy fences order the buffers' earlier generic-proxy reads and the scratch
+// rows' generic-proxy writes before the bulk copies.
 __device__ __forceinline__ void issue_tile_start(const F32View& v, ChunkPipe& pipe, float* wbuf,
-                                                 const Tile& tl, int B) {
+                                                 const Tile& tl, int B, int c0, int c1) {
     asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
     asm volatile("fence.proxy.async.global;" ::: "memory");
-    const int nchunks = (B + kPC - 1) / kPC;
-    for (int c = 0; c < nchunks && c < kNBuf; ++c)
+    for (int c = c0; c < c1 && c < c0 + kNBuf; ++c)
         issue_chunk(v, pipe, wbuf, tl.l, tl.tb, tl.cb, c, min(kPC, B - c * kPC));
+}
+
+// Balanced weight phase for large groups: when the tiles are fewer than the
+// CTAs and the group streams at least kSplitMinChunks chunks, the tiles'
+// chunks, taken in order (tile by tile) as one sequence of ntiles x nchunks,
+// are cut into gridDim.x equal runs, one per CTA.  A run is shorter than a
+// tile's chunks, so it covers at most two tiles; the CTA writes its sums for
+// each to wpart[CTA][0 or 1], and after a grid barrier weight_fixup adds each
+// tile's pieces in CTA order and applies the update.  Only for the training
+// update (fused), and only with a wpart buffer.
+constexpr int kSplitMinChunks = 24;   // measured: 16 chunks slower (the extra barrier), 32 faster
+__device__ __forceinline__ bool balanced_split(const F32View& v, int B, bool fused) {
+    return fused && v.wpart != nullptr && v.tile0[v.L + 1] < (int)gridDim.x &&
+           (B + kPC - 1) / kPC >= kSplitMinChunks;
+}
+// First flat chunk index of CTA b's run (b = gridDim.x: the end).
+__device__ __forceinline__ long long run_start(long long F, int b) { return F * b / gridDim.x; }
+
+// One weight-phase update: accumulate the change g into G (fused == false), or
+// apply lr/momentum (Section 6.2.1) after the fault guard, folding in a pending
+// G first when fold_g.
+__device__ __forceinline__ void apply_change(const F32View& v, long long idx, float g, float v_old, float g_old,
+                                             bool fused, bool fold_g) {
+    if (!fused) {
+        v.G[idx] = g_old + g;
+    } else {
+        if (fold_g) {
+            g += g_old;
+            v.G[idx] = 0.f;
+        }
+        g = guard_change(v, g);
+        const float vel = v.lr * v.grad_scale * g + v.momentum * v_old;
+        v.V[idx] = vel;
+        v.theta[idx] += vel;
+    }
 }
 
 // Pooled change of every weight (and bias: the last input column is the true
@@ -897,9 +931,14 @@ __device__ __forceinline__ void issue_tile_start(const F32View& v, ChunkPipe& pi
 // the 4 pattern lanes (butterfly), then across the 16 warps in shared memory
 // in warp order: the result does not depend on timing.
 //
+// SPLIT: the balanced form (balanced_split(v, B, fused) must hold): this
+// CTA's run of the chunk sequence, sums to wpart (a separate instantiation, so
+// that the whole-tile form keeps its registers).
+//
 // Returns false (in every thread) if a chunk copy did not arrive in time: no
 // more copies are then issued, every copy already issued has been drained, no
 // weight was written for the tile, and the caller must return.
+template <bool SPLIT>
 __device__ bool weight_phase(const F32View& v, int B, bool fused, bool fold_g, float* smem,
                              ChunkPipe& pipe) {
     const int tid = threadIdx.x;
@@ -910,7 +949,26 @@ __device__ bool weight_phase(const F32View& v, int B, bool fused, bool fold_g, f
     const int ntiles = v.tile0[L + 1];
     const int nchunks = (B + kPC - 1) / kPC;
     if (!bounds_ok(chunk_buffers_fit(v, B, wbuf), v.flags)) return true;
-    for (int t = blockIdx.x; t < ntiles; t += gridDim.x) {
+    // this CTA's work: whole tiles blockIdx.x + k gridDim.x, or (balanced) the
+    // one or two tile pieces of its run [f_lo, f_hi) of the flat chunk sequence
+    long long f_lo = 0, f_hi = 0;
+    int t_begin = blockIdx.x, t_end = ntiles, t_step = gridDim.x;
+    if constexpr (SPLIT) {
+        const long long F = (long long)ntiles * nchunks;
+        f_lo = run_start(F, blockIdx.x);
+        f_hi = run_start(F, blockIdx.x + 1);
+        t_begin = (int)(f_lo / nchunks);
+        t_end = f_hi > f_lo ? (int)((f_hi - 1) / nchunks) + 1 : t_begin;
+        t_step = 1;
+        if (!bounds_ok(t_end - t_begin <= 2, v.flags)) return true;
+    }
+    for (int t = t_begin; t < t_end; t += t_step) {
+        int c0 = 0, c1 = nchunks;
+        if constexpr (SPLIT) {
+            const long long t0 = (long long)t * nchunks;
+            c0 = (int)(max(f_lo, t0) - t0);
+            c1 = (int)(min(f_hi, t0 + nchunks) - t0);
+        }
         const Tile tl = tile_at(v, t);
         const int l = tl.l, tb = tl.tb, cb = tl.cb;
         const int n_in = v.n[l - 1], n_out = v.n[l];
@@ -920,22 +978,22 @@ __device__ bool weight_phase(const F32View& v, int B, bool fused, bool fold_g, f
         // the buffers' previous contents (weights, pattern rows, the last tile's
         // sums) were read through the generic proxy by every thread before this sync
         __syncthreads();
-        if (tid == 0) issue_tile_start(v, pipe, wbuf, tl, B);
+        if (tid == 0) issue_tile_start(v, pipe, wbuf, tl, B, c0, c1);
         // the output of threads 0..255 (unit tid / 32, column tid % 32) and its
         // current weight state, loaded now so that their latency hides behind
-        // the chunks
+        // the chunks (a piece of a balanced phase only writes its sums)
         const int uu = u0 + (tid >> 5), ii = j0 + (tid & 31);
         const bool mine = tid < kTU * kTJ && uu < n_out && ii <= n_in;
         const long long idx = v.woff[l] + (long long)uu * v.kp[l] + ii;   // ii == n_in: bias
         float v_old = 0.f, g_old = 0.f;
-        if (mine) {
+        if (mine && !SPLIT) {
             if (fused) v_old = __ldcg(v.V + idx);
             if (!fused || fold_g) g_old = __ldcg(v.G + idx);
         }
         float acc[32];   // unit u, column q of this lane's quad at u * 4 + q
 #pragma unroll
-        for (int k = 0; k < 32; ++k) acc[k] = 0.f;
-        for (int c = 0; c < nchunks; ++c) {
+        for (int q = 0; q < 32; ++q) acc[q] = 0.f;
+        for (int c = c0; c < c1; ++c) {
             const int b = c % kNBuf;
             const bool got = mbar_wait(pipe.bar + b, (pipe.parity >> b) & 1u, v.flags);
             pipe.parity ^= 1u << b;
@@ -973,15 +1031,15 @@ __device__ bool weight_phase(const F32View& v, int B, bool fused, bool fold_g, f
                 // and chunk c if thread 0 did not see it complete)
                 if (tid == 0) {
                     if (!got) mbar_drain(pipe.bar + b, ((pipe.parity >> b) & 1u) ^ 1u);
-                    for (int k = c + 1; k < nchunks && k < c + kNBuf; ++k) {
-                        const int bk = k % kNBuf;
+                    for (int c2 = c + 1; c2 < c1 && c2 < c + kNBuf; ++c2) {
+                        const int bk = c2 % kNBuf;
                         mbar_drain(pipe.bar + bk, (pipe.parity >> bk) & 1u);
                     }
                 }
                 __syncthreads();
                 return false;
             }
-            if (tid == 0 && c + kNBuf < nchunks) {
+            if (tid == 0 && c + kNBuf < c1) {
                 asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
                 issue_chunk(v, pipe, wbuf, l, tb, cb, c + kNBuf, min(kPC, B - (c + kNBuf) * kPC));
             }
@@ -990,18 +1048,18 @@ __device__ bool weight_phase(const F32View& v, int B, bool fused, bool fold_g, f
         // each level: afterwards the lane holds values base .. base + 7 (units
         // base / 4 and base / 4 + 1), base = 16 bit4 + 8 bit3
 #pragma unroll
-        for (int k = 0; k < 16; ++k) {
+        for (int q = 0; q < 16; ++q) {
             const bool up = (lane & 16) != 0;
-            const float send = up ? acc[k] : acc[k + 16];
-            const float keep = up ? acc[k + 16] : acc[k];
-            acc[k] = keep + __shfl_xor_sync(0xffffffffu, send, 16);
+            const float send = up ? acc[q] : acc[q + 16];
+            const float keep = up ? acc[q + 16] : acc[q];
+            acc[q] = keep + __shfl_xor_sync(0xffffffffu, send, 16);
         }
 #pragma unroll
-        for (int k = 0; k < 8; ++k) {
+        for (int q = 0; q < 8; ++q) {
             const bool up = (lane & 8) != 0;
-            const float send = up ? acc[k] : acc[k + 8];
-            const float keep = up ? acc[k + 8] : acc[k];
-            acc[k] = keep + __shfl_xor_sync(0xffffffffu, send, 8);
+            const float send = up ? acc[q] : acc[q + 8];
+            const float keep = up ? acc[q + 8] : acc[q];
+            acc[q] = keep + __shfl_xor_sync(0xffffffffu, send, 8);
         }
         // every warp's sums of the tile to shared memory ([warp][unit * 32 + column]);
         // the chunk buffers are free now
@@ -1017,25 +1075,48 @@ __device__ bool weight_phase(const F32View& v, int B, bool fused, bool fold_g, f
             float g = 0.f;
 #pragma unroll
             for (int w = 0; w < kWarps; ++w) g += red[w * (kTU * kTJ) + tid];
-            if (mine) {
-                if (!fused) {
-                    v.G[idx] = g_old + g;
-                } else {
-                    if (fold_g) {
-                        g += g_old;
-                        v.G[idx] = 0.f;
-                    }
-                    g = guard_change(v, g);
-                    const float vel = v.lr * v.grad_scale * g + v.momentum * v_old;
-                    v.V[idx] = vel;
-                    v.theta[idx] += vel;
-                }
+            if constexpr (SPLIT) {
+                v.wpart[((size_t)blockIdx.x * 2 + (t - t_begin)) * (kTU * kTJ) + tid] = g;
+            } else {
+                if (mine) apply_change(v, idx, g, v_old, g_old, fused, fold_g);
+                // the next group's bulk copy reads theta through the async proxy
+                asm volatile("fence.proxy.async.global;" ::: "memory");
             }
-            // the next group's bulk copy reads theta through the async proxy
-            asm volatile("fence.proxy.async.global;" ::: "memory");
         }
     }
     return true;
+}
+
+// Second step of a balanced weight phase (after a grid barrier): CTA t adds
+// the pieces of tile t in CTA order (the same order on every run) and applies
+// the update.  The CTA holding flat chunk f is the largest b with
+// floor(F b / grid) <= f, that is ((f + 1) grid - 1) / F; between the first
+// and the last CTA of a tile, CTAs with empty runs (when there are fewer
+// chunks than CTAs) hold nothing; piece k of a CTA belongs to its k-th tile.
+__device__ void weight_fixup(const F32View& v, int B, bool fold_g) {
+    const int t = blockIdx.x, tid = threadIdx.x;
+    const int ntiles = v.tile0[v.L + 1];
+    if (t >= ntiles || tid >= kTU * kTJ) return;
+    const int nchunks = (B + kPC - 1) / kPC;
+    const long long F = (long long)ntiles * nchunks, grid = gridDim.x;
+    const long long t0 = (long long)t * nchunks;
+    const int b_first = (int)(((t0 + 1) * grid - 1) / F), b_last = (int)(((t0 + nchunks) * grid - 1) / F);
+    float g = 0.f;
+    for (int b = b_first; b <= b_last; ++b) {
+        const long long start = run_start(F, b);
+        if (run_start(F, b + 1) == start) continue;   // an empty run (fewer chunks than CTAs)
+        const int k = t - (int)(start / nchunks);
+        if (bounds_ok(k >= 0 && k <= 1, v.flags)) g += __ldcg(v.wpart + ((size_t)b * 2 + k) * (kTU * kTJ) + tid);
+    }
+    const Tile tl = tile_at(v, t);
+    const int l = tl.l;
+    const int uu = tl.tb * kTU + (tid >> 5), ii = tl.cb * kTJ + (tid & 31);
+    if (uu < v.n[l] && ii <= v.n[l - 1]) {
+        const long long idx = v.woff[l] + (long long)uu * v.kp[l] + ii;
+        apply_change(v, idx, g, __ldcg(v.V + idx), fold_g ? __ldcg(v.G + idx) : 0.f, true, fold_g);
+    }
+    // the next group's bulk copy reads theta through the async proxy
+    asm volatile("fence.proxy.async.global;" ::: "memory");
 }
 
 // Initialises the weight-phase mbarriers (static shared memory) of a launch.
@@ -1139,7 +1220,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     ChunkPipe pipe;
     pipe_init(pipe, s_cbar);
     reduce_sse(v, nparts, sse_out);
-    weight_phase(v, B, false, false, smem, pipe);   // on a timeout it has drained its copies
+    weight_phase<false>(v, B, false, false, smem, pipe);   // on a timeout it has drained its copies
 }
 
 __global__ void __launch_bounds__(256) k_update(const __grid_constant__ F32View v, long long n) {
@@ -1152,7 +1233,10 @@ __global__ void __launch_bounds__(256) k_update(const __grid_constant__ F32View 
     }
 }
 
-template <int PG, bool WS>
+// SPLIT: groups that qualify (balanced_split) run the balanced weight phase;
+// a separate instantiation, chosen on the host for large minibatches, so that
+// the kernels of smaller groups carry none of its registers.
+template <int PG, bool WS, bool SPLIT>
 __global__ void __launch_bounds__(kThreads, 1)
     k_train(const __grid_constant__ F32View v, const __grid_constant__ PatLayout q, const float* X, const float* T,
             int n_patterns, int minibatch, int n_steps, float* sse_out, int fold_g) {
@@ -1192,7 +1276,15 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (threadIdx.x == 0) v.sse_part[blockIdx.x] = e;
         if (!grid_barrier(v.bar, target += gridDim.x, v.flags, wait_limit_ns(v))) return;
         reduce_sse(v, gridDim.x, sse_out != nullptr ? sse_out + s : nullptr);
-        if (!weight_phase(v, B, true, fold_g != 0 && s == 0, smem, pipe)) return;
+        bool balanced = false;
+        if constexpr (SPLIT) balanced = balanced_split(v, B, true);
+        if (balanced) {
+            if (!weight_phase<true>(v, B, true, fold_g != 0 && s == 0, smem, pipe)) return;
+            if (!grid_barrier(v.bar, target += gridDim.x, v.flags, wait_limit_ns(v))) return;
+            weight_fixup(v, B, fold_g != 0 && s == 0);
+        } else {
+            if (!weight_phase<false>(v, B, true, fold_g != 0 && s == 0, smem, pipe)) return;
+        }
         if (s + 1 < n_steps) {
             if (!grid_barrier(v.bar, target += gridDim.x, v.flags, wait_limit_ns(v))) return;
         }
@@ -1373,7 +1465,12 @@ cudaError_t set_smem_attr_ws(size_t bytes) {
     if ((e = cudaFuncSetAttribute(k_deltas<PG, WS>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                   (int)bytes)) != cudaSuccess)
         return e;
-    return cudaFuncSetAttribute(k_train<PG, WS>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+    if constexpr (PG >= 8) {
+        if ((e = cudaFuncSetAttribute(k_train<PG, WS, true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                      (int)bytes)) != cudaSuccess)
+            return e;
+    }
+    return cudaFuncSetAttribute(k_train<PG, WS, false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                 (int)bytes);
 }
 
@@ -1620,12 +1717,23 @@ cudaError_t f32_train(const F32View& v, const float* X, const float* T, int n_pa
                     (void*)&n_steps, (void*)&sse_out, (void*)&fold};
     const void* fn;
     const bool ws = plan.w_in_smem != 0;
+    // the balanced weight phase's instantiation when the minibatch qualifies
+    // (the kernel still decides per group: a ragged last group may not)
+    const bool split = v.wpart != nullptr && v.tile0[v.L + 1] < plan.grid &&
+                       (minibatch + kPC - 1) / kPC >= kSplitMinChunks;
     switch (plan.pg) {
-        case 1: fn = ws ? (const void*)k_train<1, true> : (const void*)k_train<1, false>; break;
-        case 2: fn = ws ? (const void*)k_train<2, true> : (const void*)k_train<2, false>; break;
-        case 4: fn = ws ? (const void*)k_train<4, true> : (const void*)k_train<4, false>; break;
-        case 8: fn = ws ? (const void*)k_train<8, true> : (const void*)k_train<8, false>; break;
-        default: fn = ws ? (const void*)k_train<kWidePG, true> : (const void*)k_train<kWidePG, false>; break;
+        case 1: fn = ws ? (const void*)k_train<1, true, false> : (const void*)k_train<1, false, false>; break;
+        case 2: fn = ws ? (const void*)k_train<2, true, false> : (const void*)k_train<2, false, false>; break;
+        case 4: fn = ws ? (const void*)k_train<4, true, false> : (const void*)k_train<4, false, false>; break;
+        case 8:
+            fn = split ? (ws ? (const void*)k_train<8, true, true> : (const void*)k_train<8, false, true>)
+                       : (ws ? (const void*)k_train<8, true, false> : (const void*)k_train<8, false, false>);
+            break;
+        default:
+            fn = split ? (ws ? (const void*)k_train<kWidePG, true, true> : (const void*)k_train<kWidePG, false, true>)
+                       : (ws ? (const void*)k_train<kWidePG, true, false>
+                             : (const void*)k_train<kWidePG, false, false>);
+            break;
     }
     return cudaLaunchCooperativeKernel(fn, dim3(plan.grid), dim3(kThreads), args, plan.smem, s);
 }

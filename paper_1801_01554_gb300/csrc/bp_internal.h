@@ -66,6 +66,7 @@ struct F32View {
     float* A;
     float* D;
     float* sse_part;      // one partial error sum per CTA of the pattern phase
+    float* wpart;         // balanced weight phase (large groups): [CTA][2][8 x 32] tile sums, or null
     unsigned* bar;        // grid barrier: [0] count at the end of the last launch, [1] arrival count
     int* flags;           // latched error bits
     float lr, momentum, grad_scale;

@@ -183,12 +183,16 @@ def test_train_batch_matches_oracle(sizes, B):
         check_state(sizes, theta, net.get_weights(), net.get_velocity(), st, kap, "3 updates", 3)
 
 
-def test_pending_change_is_folded_into_train_batch():
-    sizes, B = (203, 60, 26), 200
+@pytest.mark.parametrize("B,lr", [(200, 0.1), (12288, 0.01)])
+def test_pending_change_is_folded_into_train_batch(B, lr):
+    """bp_backward's pending G is added into the next training update; at
+    B = 12,288 (24 chunks) the update runs in the balanced weight phase."""
+    sizes = (203, 60, 26)
     X, T, theta = problem(sizes, B, seed=4)
     X2, T2, _ = problem(sizes, B, seed=5)
-    st = O.State(sizes, theta, lr=0.1, momentum=0.5)
-    with bp.Net(sizes, 0.1, 0.5, bp.BP_F32, max_batch=B) as net:
+    kap = [max(a, b) for a, b in zip(kappa(sizes, theta, X, T), kappa(sizes, theta, X2, T2))]
+    st = O.State(sizes, theta, lr=lr, momentum=0.5)
+    with bp.Net(sizes, lr, 0.5, bp.BP_F32, max_batch=B) as net:
         net.set_weights(theta)
         Xd = dev(X)                      # must outlive the matching bp_backward
         net.forward(Xd, B)
@@ -197,7 +201,7 @@ def test_pending_change_is_folded_into_train_batch():
         net.check()
         O.backward_accumulate(st, X, T)
         O.train_batch(st, X2, T2)
-        check_state(sizes, theta, net.get_weights(), net.get_velocity(), st, None, "folded")
+        check_state(sizes, theta, net.get_weights(), net.get_velocity(), st, kap, "folded")
         assert not net.get_grads().any()
 
 
@@ -231,6 +235,19 @@ def test_train_epoch_matches_oracle(n, mb):
         np.testing.assert_allclose(sse.cpu().numpy(), e_ref, rtol=TOL)
         check_state(sizes, theta, net.get_weights(), net.get_velocity(), st, None, "epoch",
                     len(e_ref))
+
+
+# Groups of at least 24 chunks of 512 patterns, on nets with fewer weight tiles
+# than SMs, run the balanced weight phase: each CTA takes an equal run of the
+# tiles' chunk sequence and the pieces are added in CTA order after a grid
+# barrier.  Cases: two balanced groups then a ragged one of 12 chunks in the
+# same launch; a 2-tile net (fewer chunks than CTAs, so some runs are empty);
+# exactly 24 chunks.
+@pytest.mark.parametrize("sizes,n,mb", [((203, 120, 26), 30000, 12288), ((20, 8, 3), 25500, 12500),
+                                        ((203, 60, 26), 24576, 12288)])
+def test_balanced_weight_phase_matches_oracle_step_by_step(sizes, n, mb):
+    X, T, theta = problem(sizes, n, seed=71)
+    stepwise(sizes, X, T, theta, np.zeros_like(theta), mb, 0.02, 0.9)
 
 
 @pytest.mark.parametrize("sizes,n,mb,lr", [((203, 120, 26), 777, 1, 0.05), ((203, 120, 26), 300, 1, 0.05),
@@ -326,10 +343,11 @@ def _gap_threshold(G):
     raise AssertionError("no gap")
 
 
-@pytest.mark.parametrize("B", [512, 2])
+@pytest.mark.parametrize("B", [512, 2, 16384])
 def test_fault_guard_matches_oracle(B):
-    """Section 8's guard on the persistent (B = 512) and one-CTA (B = 2) kernels:
-    the same changes are zeroed and counted, the other weights update as usual."""
+    """Section 8's guard on the persistent (B = 512), one-CTA (B = 2) and
+    balanced (B = 16,384) weight phases: the same changes are zeroed and
+    counted, the other weights update as usual."""
     sizes = (203, 120, 26)
     X, T, theta = problem(sizes, B, seed=41)
     probe = O.State(sizes, theta, lr=0.05, momentum=0.9)
