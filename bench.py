@@ -267,8 +267,8 @@ def synth_sizes(name):
 # training step (all launches) for the bf16 nets.  Re-measure after any change
 # to these kernels.
 TRAFFIC_PER_PATTERN = {
-    "nettalk60": 1_120_256 / 1024,          # 1.12 MB per launch (one update of 1,024)
-    "nettalk120": 15_591_936 / 16384,       # 62.4 MB per 65,536-pattern launch
+    "nettalk60": 1_115_392 / 1024,          # 1.12 MB per launch (one update of 1,024)
+    "nettalk120": 15_406_592 / 16384,       # 61.6 MB per 65,536-pattern launch
     "wide3": 585_467_136 / 8192,            # 585 MB per step
     "wide4096": 9_221_444_864 / 16384,      # 9.22 GB per step
 }
