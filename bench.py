@@ -523,7 +523,7 @@ def run_ours(args, world, rank, local):
     flush = torch.empty(L2_FLUSH_BYTES // 4, dtype=torch.float32, device=device)
     w = synth.WORKLOADS[WORKLOAD]
     sizes, X, T, theta = synth.make_workload(WORKLOAD, patterns=args.patterns)
-    n, mb = len(X), w["minibatch"]
+    n, mb = len(X), args.minibatch or w["minibatch"]
     epochs = w["epochs"]
     updates = -(-n // mb)
     W = connections(sizes)
@@ -566,13 +566,15 @@ def run_ours(args, world, rank, local):
     launch_s = sum(launch_ms) / len(launch_ms) / 1e3
     peak, sm_max = alu_peak_tflops(num_sms)
     achieved = algorithmic_flops_per_pattern(sizes) * n / launch_s / 1e12
-    tr = TRAFFIC_PER_PATTERN[WORKLOAD] if args.patterns is None else None
+    tr = TRAFFIC_PER_PATTERN[WORKLOAD] if args.patterns is None and args.minibatch is None else None
     line = {
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": 1e3 * dev_s_max / args.steps,
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32",
         "data": "synthetic",
-        "config": {"workload": F32_LABEL[WORKLOAD], "global_batch": mb,
+        "config": {"workload": F32_LABEL[WORKLOAD] if args.minibatch is None
+                   else F32_LABEL[WORKLOAD] + f"; minibatch {mb} for a profiler capture",
+                   "global_batch": mb,
                    "patterns_per_step": n * epochs, "updates_per_step": updates * epochs,
                    "parallelism": "replicas" if world > 1 else "single GPU",
                    "l2": "flushed (512 MB write) before every timed step"},
@@ -790,6 +792,9 @@ def main():
     ap.add_argument("--patterns", type=int, default=None,
                     help="patterns per epoch (default: the workload's; a smaller epoch of the "
                          "same net and group size is for profiler captures, not a bench line)")
+    ap.add_argument("--minibatch", type=int, default=None,
+                    help="group size of the headline net (default: the workload's 512; another "
+                         "size is for profiler captures, not a bench line)")
     ap.add_argument("--sweep", action="store_true",
                     help="instead of the bench line: CPS against the group size (203-120-26)")
     ap.add_argument("--crossover", action="store_true",
@@ -797,8 +802,8 @@ def main():
     args = ap.parse_args()
     if args.warmup < 3 and args.impl == "ours":
         args.warmup = 3
-    if args.patterns is not None:
-        args.headline_only = True      # a shortened epoch is for profiler captures only
+    if args.patterns is not None or args.minibatch is not None:
+        args.headline_only = True      # a shortened epoch or another group size: profiler captures only
     world, rank, local = dist_setup()
     if args.impl == "reference":
         rc = run_reference(args, world, rank)
