@@ -219,7 +219,7 @@ bp_status bp_create(const int* sizes, int n_layers, float lr, float momentum, in
         e = cudaMalloc(&net->A, v.a_floats * sizeof(float));
         if (e == cudaSuccess) e = cudaMalloc(&net->D, v.d_floats * sizeof(float));
         if (e == cudaSuccess) e = cudaMalloc(&net->sse_part, (size_t)net->num_sms * 4 * sizeof(float));
-        if (e == cudaSuccess) e = cudaMalloc(&net->wpart, (size_t)net->num_sms * 2 * 256 * sizeof(float));
+        if (e == cudaSuccess) e = cudaMalloc(&net->wpart, (size_t)net->num_sms * 2 * 512 * sizeof(float));
         if (e == cudaSuccess) e = cudaMalloc(&net->bar, (size_t)bp::kBarWords * sizeof(unsigned));
         if (e == cudaSuccess) e = cudaMalloc(&net->flags, 4 * sizeof(int));
         if (e != cudaSuccess) return bail(cuda_fail(e, "cudaMalloc(scratch)"));

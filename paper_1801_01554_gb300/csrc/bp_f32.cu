@@ -42,11 +42,15 @@ namespace {
 
 constexpr int kThreads = 512;
 constexpr int kWarps = kThreads / 32;
-constexpr int kTU = 8;            // weight-tile rows (output units)
+constexpr int kTU = 8;            // weight-tile rows (output units) of the whole-tile weight phase
+constexpr int kTUW = 16;          // weight-tile rows of the balanced weight phase (large groups)
+constexpr int kDB = 8;            // delta columns per scratch block
 constexpr int kTJ = 32;           // weight-tile columns (inputs; the bias is the last input)
 constexpr int kPC = 512;          // patterns per staged chunk of the weight phase
 static_assert(kPC % (kWarps * 4) == 0, "each warp takes whole groups of 4 rows of a chunk");
-constexpr int kChunkFloats = kPC * (kTU + kTJ);
+// a chunk buffer of a TU-row tile: the [kPC][kTJ] activation block, then TU / kDB delta blocks
+template <int TU>
+__host__ __device__ constexpr int chunk_floats() { return kPC * (kTJ + TU); }
 constexpr int kWarpRows = kPC / kWarps;   // rows of a chunk per warp
 // chunk buffers in flight: the CTA syncs once per chunk, so the chunk is as
 // large as two buffers allow (256 x 3 and 128 x 6 measured slower)
@@ -54,7 +58,8 @@ constexpr int kNBuf = 2;
 constexpr int kWidePG = 32;       // patterns per pass of the whole-row-per-lane forward
 // weight-phase buffers (each chunk: the [kPC][kTJ] activation block, 128-byte
 // swizzled, then the [kPC][kTU] delta block), plus room to align them to 1 KB
-constexpr size_t kGradFloats = kNBuf * kChunkFloats + 256;
+constexpr size_t kGradFloats = kNBuf * chunk_floats<kTU>() + 256;
+constexpr size_t kGradFloatsW = kNBuf * chunk_floats<kTUW>() + 256;   // balanced weight phase
 
 constexpr unsigned long long kWaitNs = 2000000000ull;   // 2 s per wait
 constexpr unsigned kWaitIters = 1u << 26;
@@ -823,40 +828,51 @@ __device__ __forceinline__ void bulk_load(float* smem_dst, const float* src, uns
                  : "memory");
 }
 
-// Weight-phase pipeline state of a CTA: kNBuf chunk buffers, each filled by two
-// TMA loads that complete on its own mbarrier; `parity` holds one phase bit per
-// buffer and persists across tiles and groups.
+// Weight-phase pipeline state of a CTA: kNBuf chunk buffers, each filled by
+// bulk copies that complete on its own mbarrier; `parity` holds one phase bit
+// per buffer and persists across tiles and groups.
 struct ChunkPipe {
     uint64_t* bar;
     unsigned parity;
 };
 
-// Issues chunk c of a tile (patterns [c * kPC, c * kPC + rows)) into buffer
-// c % kNBuf: the [rows][kTJ] activation block cb of layer l - 1, then the
-// [rows][kTU] delta block tb of layer l, each one contiguous bulk copy from the
-// blocked scratch.  Thread 0 only.
+// Issues chunk c of a TU-row tile (patterns [c * kPC, c * kPC + rows)) into
+// buffer c % kNBuf: the [rows][kTJ] activation block cb of layer l - 1, then
+// the TU / kDB delta blocks of the tile's units (blocks tb * TU / kDB ..) of
+// layer l, each one contiguous bulk copy from the blocked scratch.  Thread 0 only.
+template <int TU>
 __device__ __forceinline__ void issue_chunk(const F32View& v, ChunkPipe& pipe, float* wbuf, int l,
                                             int tb, int cb, int c, int rows) {
     const int b = c % kNBuf;
-    float* buf = wbuf + b * kChunkFloats;
-    const unsigned abytes = (unsigned)rows * kTJ * 4, dbytes = (unsigned)rows * kTU * 4;
+    float* buf = wbuf + b * chunk_floats<TU>();
+    const unsigned abytes = (unsigned)rows * kTJ * 4, dbytes = (unsigned)rows * kDB * 4;
     asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_u32(pipe.bar + b)),
-                 "r"(abytes + dbytes)
+                 "r"(abytes + (TU / kDB) * dbytes)
                  : "memory");
     const long long p0 = (long long)c * kPC;
     bulk_load(buf, v.A + v.aoff[l - 1] + (long long)cb * v.cap * kTJ + p0 * kTJ, abytes, pipe.bar + b);
-    bulk_load(buf + kPC * kTJ, v.D + v.doff[l] + (long long)tb * v.cap * kTU + p0 * kTU, dbytes, pipe.bar + b);
+#pragma unroll
+    for (int h = 0; h < TU / kDB; ++h)
+        bulk_load(buf + kPC * kTJ + h * kPC * kDB,
+                  v.D + v.doff[l] + ((long long)tb * (TU / kDB) + h) * v.cap * kDB + p0 * kDB, dbytes,
+                  pipe.bar + b);
 }
 
-// Tile t of the weight phase: its layer l, block row tb (units 8 tb ..) and
-// block column cb (inputs 32 cb ..).
+// Tile t of the weight phase (TU rows): its layer l, block row tb (units
+// TU tb ..) and block column cb (inputs 32 cb ..).
 struct Tile {
     int l, tb, cb;
 };
+template <int TU>
+__device__ __forceinline__ const int* tile_starts(const F32View& v) {
+    return TU == kTU ? v.tile0 : v.tile0w;
+}
+template <int TU>
 __device__ __forceinline__ Tile tile_at(const F32View& v, int t) {
+    const int* t0 = tile_starts<TU>(v);
     int l = 1;
-    while (t >= v.tile0[l + 1]) ++l;
-    const int lt = t - v.tile0[l];
+    while (t >= t0[l + 1]) ++l;
+    const int lt = t - t0[l];
     const int tb = lt / v.tcols[l];
     return Tile{l, tb, lt - tb * v.tcols[l]};
 }
@@ -865,32 +881,35 @@ __device__ __forceinline__ Tile tile_at(const F32View& v, int t) {
 __device__ __forceinline__ float* chunk_buffers(float* smem) {
     return reinterpret_cast<float*>((reinterpret_cast<uintptr_t>(smem) + 1023) & ~(uintptr_t)1023);
 }
+template <int TU>
 __device__ __forceinline__ bool chunk_buffers_fit(const F32View& v, int B, const float* wbuf) {
-    return (size_t)(wbuf - pattern_smem_base()) + kNBuf * kChunkFloats <= dyn_smem_floats() && B <= v.cap;
+    return (size_t)(wbuf - pattern_smem_base()) + kNBuf * chunk_floats<TU>() <= dyn_smem_floats() && B <= v.cap;
 }
 
 // Thread 0: the first kNBuf chunk copies of chunks [c0, c1) of a tile.  The
 // proxy fences order the buffers' earlier generic-proxy reads and the scratch
 // rows' generic-proxy writes before the bulk copies.
+template <int TU>
 __device__ __forceinline__ void issue_tile_start(const F32View& v, ChunkPipe& pipe, float* wbuf,
                                                  const Tile& tl, int B, int c0, int c1) {
     asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
     asm volatile("fence.proxy.async.global;" ::: "memory");
     for (int c = c0; c < c1 && c < c0 + kNBuf; ++c)
-        issue_chunk(v, pipe, wbuf, tl.l, tl.tb, tl.cb, c, min(kPC, B - c * kPC));
+        issue_chunk<TU>(v, pipe, wbuf, tl.l, tl.tb, tl.cb, c, min(kPC, B - c * kPC));
 }
 
-// Balanced weight phase for large groups: when the tiles are fewer than the
-// CTAs and the group streams at least kSplitMinChunks chunks, the tiles'
-// chunks, taken in order (tile by tile) as one sequence of ntiles x nchunks,
-// are cut into gridDim.x equal runs, one per CTA.  A run is shorter than a
-// tile's chunks, so it covers at most two tiles; the CTA writes its sums for
-// each to wpart[CTA][0 or 1], and after a grid barrier weight_fixup adds each
-// tile's pieces in CTA order and applies the update.  Only for the training
-// update (fused), and only with a wpart buffer.
+// Balanced weight phase for large groups: on tiles of kTUW rows (twice the
+// FMAs per staged byte of the whole-tile form's 8), when these tiles are fewer
+// than the CTAs and the group streams at least kSplitMinChunks chunks, the
+// tiles' chunks, taken in order (tile by tile) as one sequence of
+// ntiles x nchunks, are cut into gridDim.x equal runs, one per CTA.  A run is
+// shorter than a tile's chunks, so it covers at most two tiles; the CTA writes
+// its sums for each to wpart[CTA][0 or 1], and after a grid barrier
+// weight_fixup adds each tile's pieces in CTA order and applies the update.
+// Only for the training update (fused), and only with a wpart buffer.
 constexpr int kSplitMinChunks = 24;   // measured: 16 chunks slower (the extra barrier), 32 faster
 __device__ __forceinline__ bool balanced_split(const F32View& v, int B, bool fused) {
-    return fused && v.wpart != nullptr && v.tile0[v.L + 1] < (int)gridDim.x &&
+    return fused && v.wpart != nullptr && v.tile0w[v.L + 1] < (int)gridDim.x &&
            (B + kPC - 1) / kPC >= kSplitMinChunks;
 }
 // First flat chunk index of CTA b's run (b = gridDim.x: the end).
@@ -941,14 +960,15 @@ __device__ __forceinline__ void apply_change(const F32View& v, long long idx, fl
 template <bool SPLIT>
 __device__ bool weight_phase(const F32View& v, int B, bool fused, bool fold_g, float* smem,
                              ChunkPipe& pipe) {
+    constexpr int TU = SPLIT ? kTUW : kTU;   // tile rows
     const int tid = threadIdx.x;
     const int lane = tid & 31, warp = tid >> 5;
     const int cq = lane & 7, pl = lane >> 3;
     float* wbuf = chunk_buffers(smem);
     const int L = v.L;
-    const int ntiles = v.tile0[L + 1];
+    const int ntiles = tile_starts<TU>(v)[L + 1];
     const int nchunks = (B + kPC - 1) / kPC;
-    if (!bounds_ok(chunk_buffers_fit(v, B, wbuf), v.flags)) return true;
+    if (!bounds_ok(chunk_buffers_fit<TU>(v, B, wbuf), v.flags)) return true;
     // this CTA's work: whole tiles blockIdx.x + k gridDim.x, or (balanced) the
     // one or two tile pieces of its run [f_lo, f_hi) of the flat chunk sequence
     long long f_lo = 0, f_hi = 0;
@@ -969,60 +989,68 @@ __device__ bool weight_phase(const F32View& v, int B, bool fused, bool fold_g, f
             c0 = (int)(max(f_lo, t0) - t0);
             c1 = (int)(min(f_hi, t0 + nchunks) - t0);
         }
-        const Tile tl = tile_at(v, t);
+        const Tile tl = tile_at<TU>(v, t);
         const int l = tl.l, tb = tl.tb, cb = tl.cb;
         const int n_in = v.n[l - 1], n_out = v.n[l];
-        const int u0 = tb * kTU, j0 = cb * kTJ;
+        const int u0 = tb * TU, j0 = cb * kTJ;
         // the tile's blocks exist in the scratch layout
-        if (!bounds_ok(tb < v.dtb[l] && cb < v.acb[l - 1], v.flags)) return true;
+        if (!bounds_ok((tb + 1) * (TU / kDB) <= v.dtb[l] && cb < v.acb[l - 1], v.flags)) return true;
         // the buffers' previous contents (weights, pattern rows, the last tile's
         // sums) were read through the generic proxy by every thread before this sync
         __syncthreads();
-        if (tid == 0) issue_tile_start(v, pipe, wbuf, tl, B, c0, c1);
-        // the output of threads 0..255 (unit tid / 32, column tid % 32) and its
-        // current weight state, loaded now so that their latency hides behind
-        // the chunks (a piece of a balanced phase only writes its sums)
+        if (tid == 0) issue_tile_start<TU>(v, pipe, wbuf, tl, B, c0, c1);
+        // the output of threads 0..TU * 32 - 1 (unit tid / 32, column tid % 32)
+        // and its current weight state, loaded now so that their latency hides
+        // behind the chunks (a piece of a balanced phase only writes its sums)
         const int uu = u0 + (tid >> 5), ii = j0 + (tid & 31);
-        const bool mine = tid < kTU * kTJ && uu < n_out && ii <= n_in;
+        const bool mine = tid < TU * kTJ && uu < n_out && ii <= n_in;
         const long long idx = v.woff[l] + (long long)uu * v.kp[l] + ii;   // ii == n_in: bias
         float v_old = 0.f, g_old = 0.f;
         if (mine && !SPLIT) {
             if (fused) v_old = __ldcg(v.V + idx);
             if (!fused || fold_g) g_old = __ldcg(v.G + idx);
         }
-        float acc[32];   // unit u, column q of this lane's quad at u * 4 + q
+        float acc[TU * 4];   // unit u, column q of this lane's quad at u * 4 + q
 #pragma unroll
-        for (int q = 0; q < 32; ++q) acc[q] = 0.f;
+        for (int q = 0; q < TU * 4; ++q) acc[q] = 0.f;
         for (int c = c0; c < c1; ++c) {
             const int b = c % kNBuf;
             const bool got = mbar_wait(pipe.bar + b, (pipe.parity >> b) & 1u, v.flags);
             pipe.parity ^= 1u << b;
-            float* As = wbuf + b * kChunkFloats;
-            float* Ds = As + kPC * kTJ;
+            float* As = wbuf + b * chunk_floats<TU>();
+            float* Ds = As + kPC * kTJ;   // TU / kDB delta blocks of [kPC][kDB]
             const int pc = B - c * kPC;
             if (pc < kPC) {
                 // rows past the group may hold stale scratch rows: clear those
                 // in the share of the last warp with live rows (the warps after
                 // it skip the chunk)
                 const int pend = min(kPC, (pc + kWarpRows - 1) / kWarpRows * kWarpRows);
-                for (int e = tid; e < (pend - pc) * kTU; e += kThreads) Ds[pc * kTU + e] = 0.f;
+#pragma unroll
+                for (int h = 0; h < TU / kDB; ++h)
+                    for (int e = tid; e < (pend - pc) * kDB; e += kThreads) Ds[h * kPC * kDB + pc * kDB + e] = 0.f;
                 for (int e = tid; e < (pend - pc) * kTJ; e += kThreads) As[pc * kTJ + e] = 0.f;
                 __syncthreads();
             }
             if (warp * kWarpRows < pc) {   // warp-uniform: the warp has live rows
-#pragma unroll
+                // (the 16-row form unrolls less: its 64 sums leave fewer registers)
+#pragma unroll(TU == kTU ? kWarpRows / 4 : 2)
                 for (int i = 0; i < kWarpRows / 4; ++i) {
                     const int p = warp * kWarpRows + 4 * i + pl;   // row of the chunk
                     const int dsw = (p >> 2) & 1;
-                    const float4 d0 = *reinterpret_cast<const float4*>(Ds + p * kTU + (dsw << 2));
-                    const float4 d1 = *reinterpret_cast<const float4*>(Ds + p * kTU + ((1 ^ dsw) << 2));
                     const float4 a = *reinterpret_cast<const float4*>(As + p * kTJ + ((cq ^ (p & 7)) << 2));
-                    const float dv[8] = {d0.x, d0.y, d0.z, d0.w, d1.x, d1.y, d1.z, d1.w};
                     const float av[4] = {a.x, a.y, a.z, a.w};
 #pragma unroll
-                    for (int u = 0; u < 8; ++u)
+                    for (int h = 0; h < TU / kDB; ++h) {   // one delta block (8 units) at a time
+                        const float* Dh = Ds + h * kPC * kDB + p * kDB;
+                        const float4 d0 = *reinterpret_cast<const float4*>(Dh + (dsw << 2));
+                        const float4 d1 = *reinterpret_cast<const float4*>(Dh + ((1 ^ dsw) << 2));
+                        const float dv[8] = {d0.x, d0.y, d0.z, d0.w, d1.x, d1.y, d1.z, d1.w};
 #pragma unroll
-                        for (int q = 0; q < 4; ++q) acc[u * 4 + q] = fmaf(dv[u], av[q], acc[u * 4 + q]);
+                        for (int u = 0; u < 8; ++u)
+#pragma unroll
+                            for (int q = 0; q < 4; ++q)
+                                acc[(h * 8 + u) * 4 + q] = fmaf(dv[u], av[q], acc[(h * 8 + u) * 4 + q]);
+                    }
                 }
             }
             if (__syncthreads_or(!got)) {
@@ -1041,42 +1069,43 @@ __device__ bool weight_phase(const F32View& v, int B, bool fused, bool fold_g, f
             }
             if (tid == 0 && c + kNBuf < c1) {
                 asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-                issue_chunk(v, pipe, wbuf, l, tb, cb, c + kNBuf, min(kPC, B - (c + kNBuf) * kPC));
+                issue_chunk<TU>(v, pipe, wbuf, l, tb, cb, c + kNBuf, min(kPC, B - (c + kNBuf) * kPC));
             }
         }
         // sum over the 4 pattern lanes (lane bits 4, 3), halving the values at
-        // each level: afterwards the lane holds values base .. base + 7 (units
-        // base / 4 and base / 4 + 1), base = 16 bit4 + 8 bit3
+        // each level: afterwards the lane holds values 0 .. TU - 1 of units
+        // ub .. ub + TU / 4 - 1, ub = TU / 2 bit4 + TU / 4 bit3 (each sum is
+        // (lane 0 + lane 2) + (lane 1 + lane 3) of the pattern lanes)
 #pragma unroll
-        for (int q = 0; q < 16; ++q) {
+        for (int q = 0; q < TU * 2; ++q) {
             const bool up = (lane & 16) != 0;
-            const float send = up ? acc[q] : acc[q + 16];
-            const float keep = up ? acc[q + 16] : acc[q];
+            const float send = up ? acc[q] : acc[q + TU * 2];
+            const float keep = up ? acc[q + TU * 2] : acc[q];
             acc[q] = keep + __shfl_xor_sync(0xffffffffu, send, 16);
         }
 #pragma unroll
-        for (int q = 0; q < 8; ++q) {
+        for (int q = 0; q < TU; ++q) {
             const bool up = (lane & 8) != 0;
-            const float send = up ? acc[q] : acc[q + 8];
-            const float keep = up ? acc[q + 8] : acc[q];
+            const float send = up ? acc[q] : acc[q + TU];
+            const float keep = up ? acc[q + TU] : acc[q];
             acc[q] = keep + __shfl_xor_sync(0xffffffffu, send, 8);
         }
         // every warp's sums of the tile to shared memory ([warp][unit * 32 + column]);
         // the chunk buffers are free now
         float* red = wbuf;
-        const int ub = ((lane >> 4) & 1) * 4 + ((lane >> 3) & 1) * 2;   // first of this lane's two units
+        const int ub = ((lane >> 4) & 1) * (TU / 2) + ((lane >> 3) & 1) * (TU / 4);
         __syncthreads();
-        *reinterpret_cast<float4*>(red + warp * (kTU * kTJ) + ub * kTJ + 4 * cq) =
-            make_float4(acc[0], acc[1], acc[2], acc[3]);
-        *reinterpret_cast<float4*>(red + warp * (kTU * kTJ) + (ub + 1) * kTJ + 4 * cq) =
-            make_float4(acc[4], acc[5], acc[6], acc[7]);
+#pragma unroll
+        for (int i = 0; i < TU / 4; ++i)
+            *reinterpret_cast<float4*>(red + warp * (TU * kTJ) + (ub + i) * kTJ + 4 * cq) =
+                make_float4(acc[4 * i], acc[4 * i + 1], acc[4 * i + 2], acc[4 * i + 3]);
         __syncthreads();
-        if (tid < kTU * kTJ) {
+        if (tid < TU * kTJ) {
             float g = 0.f;
 #pragma unroll
-            for (int w = 0; w < kWarps; ++w) g += red[w * (kTU * kTJ) + tid];
+            for (int w = 0; w < kWarps; ++w) g += red[w * (TU * kTJ) + tid];
             if constexpr (SPLIT) {
-                v.wpart[((size_t)blockIdx.x * 2 + (t - t_begin)) * (kTU * kTJ) + tid] = g;
+                v.wpart[((size_t)blockIdx.x * 2 + (t - t_begin)) * (kTUW * kTJ) + tid] = g;
             } else {
                 if (mine) apply_change(v, idx, g, v_old, g_old, fused, fold_g);
                 // the next group's bulk copy reads theta through the async proxy
@@ -1095,8 +1124,8 @@ __device__ bool weight_phase(const F32View& v, int B, bool fused, bool fold_g, f
 // chunks than CTAs) hold nothing; piece k of a CTA belongs to its k-th tile.
 __device__ void weight_fixup(const F32View& v, int B, bool fold_g) {
     const int t = blockIdx.x, tid = threadIdx.x;
-    const int ntiles = v.tile0[v.L + 1];
-    if (t >= ntiles || tid >= kTU * kTJ) return;
+    const int ntiles = v.tile0w[v.L + 1];
+    if (t >= ntiles || tid >= kTUW * kTJ) return;
     const int nchunks = (B + kPC - 1) / kPC;
     const long long F = (long long)ntiles * nchunks, grid = gridDim.x;
     const long long t0 = (long long)t * nchunks;
@@ -1106,11 +1135,11 @@ __device__ void weight_fixup(const F32View& v, int B, bool fold_g) {
         const long long start = run_start(F, b);
         if (run_start(F, b + 1) == start) continue;   // an empty run (fewer chunks than CTAs)
         const int k = t - (int)(start / nchunks);
-        if (bounds_ok(k >= 0 && k <= 1, v.flags)) g += __ldcg(v.wpart + ((size_t)b * 2 + k) * (kTU * kTJ) + tid);
+        if (bounds_ok(k >= 0 && k <= 1, v.flags)) g += __ldcg(v.wpart + ((size_t)b * 2 + k) * (kTUW * kTJ) + tid);
     }
-    const Tile tl = tile_at(v, t);
+    const Tile tl = tile_at<kTUW>(v, t);
     const int l = tl.l;
-    const int uu = tl.tb * kTU + (tid >> 5), ii = tl.cb * kTJ + (tid & 31);
+    const int uu = tl.tb * kTUW + (tid >> 5), ii = tl.cb * kTJ + (tid & 31);
     if (uu < v.n[l] && ii <= v.n[l - 1]) {
         const long long idx = v.woff[l] + (long long)uu * v.kp[l] + ii;
         apply_change(v, idx, g, __ldcg(v.V + idx), fold_g ? __ldcg(v.G + idx) : 0.f, true, fold_g);
@@ -1493,9 +1522,10 @@ long long f32_layout(F32View& v, const int* n, int L, int cap) {
     v.L = L;
     v.cap = cap;
     long long pos = 0, a = 0, d = 0;
-    int tiles = 0;
+    int tiles = 0, tiles_w = 0;
     for (int l = 0; l <= L; ++l) v.n[l] = n[l];
     v.tile0[0] = v.tile0[1] = 0;
+    v.tile0w[0] = v.tile0w[1] = 0;
     for (int l = 0; l <= L; ++l) {
         v.apitch[l] = (n[l] + 1 + 3) & ~3;
         v.acb[l] = (n[l] + 1 + kTJ - 1) / kTJ;
@@ -1512,14 +1542,18 @@ long long f32_layout(F32View& v, const int* n, int L, int cap) {
         v.pb[l] = pp;
         pp += n[l];
         v.dpitch[l] = (n[l] + 3) & ~3;
-        v.dtb[l] = (n[l] + kTU - 1) / kTU;
+        // an even number of delta blocks, so that a kTUW-row tile always has its two
+        v.dtb[l] = ((n[l] + kDB - 1) / kDB + 1) & ~1;
         v.doff[l] = d;
-        d += (long long)cap * v.dtb[l] * kTU;
+        d += (long long)cap * v.dtb[l] * kDB;
         const int rows = (n[l] + kTU - 1) / kTU, cols = (n[l - 1] + 1 + kTJ - 1) / kTJ;
         v.tcols[l] = cols;
         v.tile0[l] = tiles;
         tiles += rows * cols;
         v.tile0[l + 1] = tiles;
+        v.tile0w[l] = tiles_w;
+        tiles_w += ((n[l] + kTUW - 1) / kTUW) * cols;
+        v.tile0w[l + 1] = tiles_w;
     }
     v.P = pos;   // a multiple of 4: every kp is
     v.Pp = pp;
@@ -1639,7 +1673,15 @@ F32Plan f32_plan(const F32View& v, int batch, int num_sms) {
     const size_t pat = pattern_floats(v.n, v.L, pg);
     p.w_in_smem = (((size_t)v.wsm + pat) * sizeof(float) <= kSmemLimit) ? 1 : 0;
     size_t need = p.w_in_smem ? (size_t)v.wsm + pat : pat;
-    if (need < (size_t)kGradFloats) need = kGradFloats;
+    // the balanced weight phase (and its larger chunk buffers) when the
+    // minibatch qualifies; the kernel still decides per group (a ragged last
+    // group may not)
+    p.split = (v.wpart != nullptr && v.tile0w[v.L + 1] < num_sms && (batch + kPC - 1) / kPC >= kSplitMinChunks &&
+               pg >= 8 && (size_t)kGradFloatsW * sizeof(float) <= kSmemLimit)
+                  ? 1
+                  : 0;
+    const size_t grad = p.split ? kGradFloatsW : kGradFloats;
+    if (need < grad) need = grad;
     p.smem = need * sizeof(float);
     p.q = pat_layout(v.n, v.L, pg);
     return p;
@@ -1717,10 +1759,7 @@ cudaError_t f32_train(const F32View& v, const float* X, const float* T, int n_pa
                     (void*)&n_steps, (void*)&sse_out, (void*)&fold};
     const void* fn;
     const bool ws = plan.w_in_smem != 0;
-    // the balanced weight phase's instantiation when the minibatch qualifies
-    // (the kernel still decides per group: a ragged last group may not)
-    const bool split = v.wpart != nullptr && v.tile0[v.L + 1] < plan.grid &&
-                       (minibatch + kPC - 1) / kPC >= kSplitMinChunks;
+    const bool split = plan.split != 0;
     switch (plan.pg) {
         case 1: fn = ws ? (const void*)k_train<1, true, false> : (const void*)k_train<1, false, false>; break;
         case 2: fn = ws ? (const void*)k_train<2, true, false> : (const void*)k_train<2, false, false>; break;

@@ -34,12 +34,14 @@ constexpr int kBarWords = 4;
 //      pattern's 128-byte block row the 16-byte chunk k sits at k ^ (p mod 8),
 //      so that the weight phase's lanes read 32 consecutive rows without bank
 //      conflicts; a chunk of a tile is one contiguous bulk copy.
-//   D: deltas of layers 1..L at doff[l] in dtb[l] blocks of [cap][8] floats,
-//      chunk k of a 32-byte block row at k ^ ((p / 4) mod 2).
+//   D: deltas of layers 1..L at doff[l] in dtb[l] blocks of [cap][8] floats
+//      (an even number of blocks per layer), chunk k of a 32-byte block row at
+//      k ^ ((p / 4) mod 2).
 //   apitch[l] = n_l + 1 and dpitch[l] = n_l rounded up to 4 are the row
 //   pitches of the same rows in shared memory.
 //   Gradient tiles: layer l owns tiles [tile0[l], tile0[l+1]) of 8 rows x 32
-//   columns of the [n_l, n_{l-1} + 1] matrix (last column = bias).
+//   columns of the [n_l, n_{l-1} + 1] matrix (last column = bias), and tiles
+//   [tile0w[l], tile0w[l+1]) of 16 rows x 32 columns in the balanced form.
 struct F32View {
     int L;
     int cap;
@@ -59,6 +61,7 @@ struct F32View {
     long long doff[BP_MAX_SIZES];
     long long a_floats, d_floats;
     int tile0[BP_MAX_SIZES + 1];
+    int tile0w[BP_MAX_SIZES + 1];  // the same for the balanced weight phase's 16-row tiles
     int tcols[BP_MAX_SIZES];
     float* theta;
     float* V;
@@ -66,7 +69,7 @@ struct F32View {
     float* A;
     float* D;
     float* sse_part;      // one partial error sum per CTA of the pattern phase
-    float* wpart;         // balanced weight phase (large groups): [CTA][2][8 x 32] tile sums, or null
+    float* wpart;         // balanced weight phase (large groups): [CTA][2][16 x 32] tile sums, or null
     unsigned* bar;        // grid barrier: [0] count at the end of the last launch, [1] arrival count
     int* flags;           // latched error bits
     float lr, momentum, grad_scale;
@@ -96,6 +99,7 @@ struct F32Plan {
     int w_in_smem;   // the weights are copied into shared memory
     size_t smem;     // dynamic shared memory bytes
     PatLayout q;     // pattern buffers
+    int split;       // training launches use the balanced weight phase (large minibatches)
 };
 
 // --- float32 path (bp_f32.cu) -------------------------------------------
