@@ -952,12 +952,28 @@ bool alloc(Bf16Net* b, void** p, size_t bytes) {
 
 int ceil_div(long long a, long long b) { return (int)((a + b - 1) / b); }
 
+// Splits of K (the batch) for a pooled-change GEMM of `tiles` output tiles:
+// the fewest that minimise, in units of one full-K tile's time on one SM,
+//   ceil(tiles * s / num_sms) / s     (waves of 1/s-K work items)
+//   + s * r                           (the s partial planes: written here, read by the update)
+// with r = (tile bytes of fp32 partials, out and back) / (tile MMA time) =
+// 8 BM BN / HBM  /  (2 BM BN K / (bf16 peak / SM)) = 4 F_sm / (K HBM); the
+// measured ratio of per-SM bf16 peak to HBM bandwidth, 12.7 TFLOP/s to
+// 6.8 TB/s, is 1.87 flop per byte.
 int pick_splits(int tiles, int kb_total, int num_sms, int cap_splits) {
-    int s = num_sms / (tiles > 0 ? tiles : 1);
-    if (s < 1) s = 1;
-    if (s > cap_splits) s = cap_splits;
-    if (s > kb_total) s = kb_total;
-    return s;
+    if (tiles < 1) tiles = 1;
+    const double r = 4.0 * 1.87 / ((double)kb_total * BK);
+    int best = 1;
+    double best_cost = 0.0;
+    for (int s = 1; s <= cap_splits && s <= kb_total; ++s) {
+        const double waves = (double)(((long long)tiles * s + num_sms - 1) / num_sms) / s;
+        const double cost = waves + s * r * tiles;
+        if (s == 1 || cost < best_cost * (1.0 - 1e-9)) {
+            best = s;
+            best_cost = cost;
+        }
+    }
+    return best;
 }
 
 template <int MODE>
