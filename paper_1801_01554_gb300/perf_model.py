@@ -79,30 +79,43 @@ def gf11_optimal_processors(W, Wi, U, C, summing="tree", M=GF11_FREE_SRAM, bundl
 # ---------------------------------------------------------------- GB300 restatement
 @dataclass
 class GB300Phases:
-    """Phase costs of the float32 kernels on one GB300 (microseconds), measured
-    for the 203-120-26 net with each phase looped inside one launch."""
+    """Phase costs of the float32 kernels on one GB300 (microseconds), fitted
+    to per-update times of the 203-120-26 net with and without the weight
+    phase (a timing-only copy of the kernel) at B = 8 .. 65,536."""
     n_sm: int = 152
-    barrier_us: float = 1.29          # one grid barrier (two per update)
-    weight_copy_us: float = 0.70      # 110.8 KB bulk copy into each CTA's shared memory
-    # one pattern pass of PG patterns on a CTA (rows, forward, deltas, rows out)
-    pass_us: tuple = ((1, 4.11), (2, 4.44), (4, 5.30), (8, 7.86))
-    chunk_us: float = 0.744           # one 256-pattern chunk of a weight tile
-    weight_fixed_us: float = 1.35     # chunk issue, tile reduction and update
-    skew_us: float = 0.86             # arrival skew between CTAs, the remainder at B = 512
+    # pattern side of an update: two grid barriers, the weight copy, skew, and
+    # one pass per PG patterns of a CTA's share
+    pattern_fixed_us: float = 4.79
+    pass_us: tuple = ((1, 3.10), (2, 3.43), (4, 4.56), (8, 7.09), (32, 16.3))
+    # whole-tile weight phase (8 x 32 tiles, one per CTA): fixed part, then per
+    # 512-pattern chunk a fixed and a per-row part
+    weight_fixed_us: float = 1.27
+    chunk_fixed_us: float = 0.58
+    chunk_rows_us: float = 0.72        # for a full chunk of 512 rows
+    # balanced weight phase (16 x 32 tiles, equal runs of chunks per CTA, one
+    # more grid barrier and the fix-up): fixed part and per chunk of a run
+    balanced_fixed_us: float = 6.66
+    balanced_chunk_us: float = 2.23
+    balanced_min_chunks: int = 24
+    chunk_rows: int = 512
     # one-CTA kernel: per group of B patterns
     small_us: tuple = ((1, 6.68), (2, 7.37), (4, 9.17))
 
 
-def gb300_group_size(B, n_sm=152, max_pg=8):
-    """Patterns per CTA pass (PG) that the persistent kernel picks for B."""
+def gb300_group_size(B, n_sm=152, max_pg=8, wide=True):
+    """Patterns per CTA pass (PG) that the persistent kernel picks for B:
+    doubling up to 8, then passes of 32 above 16 patterns per CTA when the
+    net suits them (wide; true for 203-120-26)."""
     want = -(-B // n_sm)
     pg = 1
     while pg < want and pg < max_pg:
         pg *= 2
+    if wide and want > 16 and pg == 8:
+        pg = 32
     return pg
 
 
-def gb300_update_us(B, tiles=121, ph: GB300Phases = GB300Phases(), small_max=4):
+def gb300_update_us(B, tiles=121, tiles16=64, ph: GB300Phases = GB300Phases(), small_max=4):
     """Predicted microseconds per update of a B-pattern group (203-120-26)."""
     if B <= small_max:
         for b, us in ph.small_us:
@@ -110,10 +123,16 @@ def gb300_update_us(B, tiles=121, ph: GB300Phases = GB300Phases(), small_max=4):
                 return us
     pg = gb300_group_size(B, ph.n_sm)
     passes = -(-(-(-B // ph.n_sm)) // pg)
-    t_pass = dict(ph.pass_us)[pg]
-    chunks = -(-B // 256) * -(-tiles // ph.n_sm)
-    return (2 * ph.barrier_us + ph.weight_copy_us + passes * t_pass + chunks * ph.chunk_us
-            + ph.weight_fixed_us + ph.skew_us)
+    t = ph.pattern_fixed_us + passes * dict(ph.pass_us)[pg]
+    chunks = -(-B // ph.chunk_rows)
+    if chunks >= ph.balanced_min_chunks and tiles16 < ph.n_sm:
+        run = -(-(tiles16 * chunks) // ph.n_sm)
+        return t + ph.balanced_fixed_us + run * ph.balanced_chunk_us
+    per_cta = -(-tiles // ph.n_sm)
+    rows_last = B - (chunks - 1) * ph.chunk_rows
+    w = ph.weight_fixed_us + per_cta * ((chunks - 1) * (ph.chunk_fixed_us + ph.chunk_rows_us)
+                                        + ph.chunk_fixed_us + ph.chunk_rows_us * rows_last / ph.chunk_rows)
+    return t + w
 
 
 def gb300_cps(B, W=27626, **kw):

@@ -56,11 +56,14 @@ def test_tree_beats_ring_beyond_a_few_processors():
 
 
 def test_gb300_model_is_monotone_and_uses_the_kernels_group_sizes():
-    Bs = [1, 2, 3, 4, 5, 8, 64, 152, 153, 512, 1216, 1217, 4096, 65536]
+    Bs = [1, 2, 3, 4, 5, 8, 64, 152, 153, 512, 1216, 1217, 2432, 2433, 4096, 12288, 65536]
     t = [M.gb300_update_us(b) for b in Bs]
     assert all(b >= a for a, b in zip(t, t[1:]))
     assert M.gb300_group_size(512) == 4 and M.gb300_group_size(152) == 1
-    assert M.gb300_group_size(153) == 2 and M.gb300_group_size(65536) == 8
+    assert M.gb300_group_size(153) == 2 and M.gb300_group_size(2432) == 8
+    # passes of 32 from 17 patterns per CTA on (the kernel's rule for the NETtalk shapes)
+    assert M.gb300_group_size(2433) == 32 and M.gb300_group_size(65536) == 32
+    assert M.gb300_group_size(65536, wide=False) == 8
     # over powers of two CPS grows with the group size: the fixed cost of an
     # update is amortised (a ragged extra pass can lower it in between)
     cps = [M.gb300_cps(2 ** k) for k in range(17)]
