@@ -272,6 +272,9 @@ TRAFFIC_PER_PATTERN = {
     "wide3": 585_467_136 / 8192,            # 585 MB per step
     "wide4096": 9_221_444_864 / 16384,      # 9.22 GB per step
 }
+# sweep groups of 203-120-26 with a capture of their own (bytes per pattern of one launch);
+# at B = 65,536 the group's scratch rows no longer fit the L2 and make a DRAM round trip
+SWEEP_TRAFFIC_PER_PATTERN = {512: TRAFFIC_PER_PATTERN["nettalk120"], 65536: 594_142_976 / 65536}
 
 
 def connections(sizes):
@@ -623,7 +626,10 @@ def run_ours(args, world, rank, local):
             c = cpu.get(("sweep", B))
             sweep.append({"B": B, "patterns": nb, "value": ent["value"],
                           "us_per_update": 1e3 * ent["ms_per_step"] / -(-nb // B),
-                          "frac": ent["roofline"]["frac"], "e2e": ent["e2e"]["value"],
+                          "frac": ent["roofline"]["frac"],
+                          "traffic": (SWEEP_TRAFFIC_PER_PATTERN[B] * nb if B in SWEEP_TRAFFIC_PER_PATTERN
+                                      else None),
+                          "e2e": ent["e2e"]["value"],
                           "cpu_one_core": c["one_core"] if c else None,
                           "cpu_all_cores": c["value"] if c else None,
                           "cpu_cores": c["cores"] if c else None})
