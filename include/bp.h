@@ -209,8 +209,9 @@ bp_status bp_train_epoch(bp_net* net, const void* d_X, const void* d_T, int n_pa
  * minibatch) error sums back to h_sse (may be NULL) and waits for the stream.
  * The epoch runs in up to 8 pieces of whole minibatches, each copied on a
  * stream of the net's own while the previous piece trains (the copies overlap
- * compute when h_X and h_T are pinned); the updates are the same as one
- * bp_train_epoch over the whole pass.
+ * compute when h_X and h_T are pinned); pieces double from ceil(groups / 128)
+ * minibatches, so that little of the copy waits in front of the first
+ * update.  The updates are the same as one bp_train_epoch over the whole pass.
  * Errors as bp_train_epoch, plus BP_ENOMEM for the staging buffers and any
  * error latched by the epoch's kernels (as bp_check). */
 bp_status bp_train_epoch_host(bp_net* net, const void* h_X, const void* h_T, int n_patterns,

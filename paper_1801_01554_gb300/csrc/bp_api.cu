@@ -569,20 +569,22 @@ bp_status bp_train_epoch_host(bp_net* net, const void* h_X, const void* h_T, int
     }
     // The epoch runs in up to 8 pieces of whole minibatches: the copy of piece
     // k + 1 (on the net's copy stream) overlaps the training of piece k (on the
-    // caller's stream), which waits for its own piece only.  The staging
-    // buffers may still be read by work queued earlier on the caller's stream.
+    // caller's stream), which waits for its own piece only.  Pieces double in
+    // size from f = ceil(steps / 128) minibatches (f, 2f, .. 64f, then the rest,
+    // at most f), so that only 1/128 of the epoch's copy is exposed and no copy
+    // is more than twice the training it hides behind.  The staging buffers may
+    // still be read by work queued earlier on the caller's stream.
     BP_CUDA(cudaEventRecord(net->start_ev, s), "copy events");
     BP_CUDA(cudaStreamWaitEvent(net->copy_stream, net->start_ev, 0), "copy events");
     const long long n_steps = (long long)ns;
-    const int pieces = (int)(n_steps < 8 ? n_steps : 8);
-    const long long per = (n_steps + pieces - 1) / pieces;
     const size_t xrow = (size_t)net->n[0] * elem_size(net);
     const size_t trow = (size_t)net->n[net->L] * elem_size(net);
-    for (int k = 0; k < pieces; ++k) {
-        const long long step0 = k * per;
-        if (step0 >= n_steps) break;
+    const long long first = (n_steps + 127) / 128;
+    long long step0 = 0;
+    for (int k = 0; k < 8 && step0 < n_steps; ++k) {
+        const long long steps_k = k == 7 ? n_steps - step0 : std::min(first << k, n_steps - step0);
         const long long p0 = step0 * minibatch;
-        const long long np = std::min((long long)n_patterns - p0, per * minibatch);
+        const long long np = std::min((long long)n_patterns - p0, steps_k * minibatch);
         char* dx = (char*)net->stage_X + p0 * xrow;
         char* dt = (char*)net->stage_T + p0 * trow;
         BP_CUDA(cudaMemcpyAsync(dx, (const char*)h_X + p0 * xrow, np * xrow, cudaMemcpyHostToDevice,
@@ -595,6 +597,7 @@ bp_status bp_train_epoch_host(bp_net* net, const void* h_X, const void* h_T, int
         BP_CUDA(cudaStreamWaitEvent(s, net->piece_ev[k], 0), "copy events");
         st = run_epoch(net, dx, dt, (int)np, minibatch, net->stage_sse + step0, s);
         if (st != BP_OK) return st;
+        step0 += steps_k;
     }
     if (h_sse != nullptr)
         BP_CUDA(cudaMemcpyAsync(h_sse, net->stage_sse, ns * sizeof(float), cudaMemcpyDeviceToHost, s),
