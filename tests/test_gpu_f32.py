@@ -237,6 +237,16 @@ def test_train_epoch_matches_oracle(n, mb):
                     len(e_ref))
 
 
+def test_weights_beyond_shared_memory_at_large_groups_step_by_step():
+    """203-512-26 in groups of 4,096: 460 KB of padded weights do not fit in
+    shared memory, so the pattern passes (of 8: passes of 32 need the weights
+    in shared memory) read them from global memory, and its 516 weight tiles
+    are more than the CTAs (each CTA takes several in turn)."""
+    sizes = (203, 512, 26)
+    X, T, theta = problem(sizes, 8192, seed=81, lo=-0.3, hi=0.3)
+    stepwise(sizes, X, T, theta, np.zeros_like(theta), 4096, 0.01, 0.9)
+
+
 # Groups of at least 24 chunks of 512 patterns, on nets with fewer weight tiles
 # than SMs, run the balanced weight phase: each CTA takes an equal run of the
 # tiles' chunk sequence and the pieces are added in CTA order after a grid
@@ -281,7 +291,8 @@ def test_one_launch_epoch_is_reproducible():
     assert np.array_equal(runs[0][0], runs[1][0]) and np.array_equal(runs[0][1], runs[1][1])
 
 
-@pytest.mark.parametrize("sizes,n,mb", [((203, 120, 26), 1024, 512), ((64, 33, 17, 9), 257, 256)])
+@pytest.mark.parametrize("sizes,n,mb", [((203, 120, 26), 1024, 512), ((64, 33, 17, 9), 257, 256),
+                                        ((203, 120, 26), 8192, 4096)])   # passes of 32
 def test_table_sigmoid_matches_oracle(sizes, n, mb):
     """The table-lookup logistic of Section 4.3 on the persistent kernel: the
     outputs of a forward pass and an epoch of updates against the oracle's
