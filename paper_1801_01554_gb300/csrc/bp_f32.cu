@@ -829,11 +829,15 @@ __device__ __forceinline__ void bulk_load(float* smem_dst, const float* src, uns
 }
 
 // Weight-phase pipeline state of a CTA: kNBuf chunk buffers, each filled by
-// bulk copies that complete on its own mbarrier; `parity` holds one phase bit
-// per buffer and persists across tiles and groups.
+// bulk copies that complete on its own "full" mbarrier, and released by the
+// 16 warps on its own "empty" mbarrier (one arrival per warp) before thread 0
+// refills it; `parity` and `eparity` hold one phase bit per buffer and persist
+// across tiles and groups.
 struct ChunkPipe {
     uint64_t* bar;
     unsigned parity;
+    uint64_t* ebar;      // per buffer: all warps done with it (thread 0 waits)
+    unsigned eparity;    // thread 0's
 };
 
 // Issues chunk c of a TU-row tile (patterns [c * kPC, c * kPC + rows)) into
@@ -946,17 +950,20 @@ __device__ __forceinline__ void apply_change(const F32View& v, long long idx, fl
 // delta loads shared by the 8 lanes of a pattern lane and one 16-byte
 // activation load for 32 FMAs, which keeps the loop off the shared-memory
 // bandwidth limit.  The blocks' row chunks are stored permuted by pattern (see
-// F32View), so the lanes' reads are conflict-free.  The sums meet first across
-// the 4 pattern lanes (butterfly), then across the 16 warps in shared memory
-// in warp order: the result does not depend on timing.
+// F32View), so the lanes' reads are conflict-free.  There is no CTA-wide sync
+// per chunk: each warp releases a buffer on its empty barrier and thread 0
+// refills it once all have, so warps may run up to a chunk apart (a CTA sync
+// per chunk measured 1-2% slower).  The sums meet first across the 4 pattern
+// lanes (butterfly), then across the 16 warps in shared memory in warp order:
+// the result does not depend on timing.
 //
 // SPLIT: the balanced form (balanced_split(v, B, fused) must hold): this
 // CTA's run of the chunk sequence, sums to wpart (a separate instantiation, so
 // that the whole-tile form keeps its registers).
 //
-// Returns false (in every thread) if a chunk copy did not arrive in time: no
-// more copies are then issued, every copy already issued has been drained, no
-// weight was written for the tile, and the caller must return.
+// Returns false (in every thread) if a wait ran out: thread 0 then issues no
+// more copies and has waited for (or drained) every copy it issued, no weight
+// was written for the tile, and the caller must return.
 template <bool SPLIT>
 __device__ bool weight_phase(const F32View& v, int B, bool fused, bool fold_g, float* smem,
                              ChunkPipe& pipe) {
@@ -1013,25 +1020,31 @@ __device__ bool weight_phase(const F32View& v, int B, bool fused, bool fold_g, f
         float acc[TU * 4];   // unit u, column q of this lane's quad at u * 4 + q
 #pragma unroll
         for (int q = 0; q < TU * 4; ++q) acc[q] = 0.f;
+        bool all_got = true;   // this thread's waits all arrived
+        bool stop = false;     // thread 0: a wait ran out, no more copies
         for (int c = c0; c < c1; ++c) {
             const int b = c % kNBuf;
-            const bool got = mbar_wait(pipe.bar + b, (pipe.parity >> b) & 1u, v.flags);
+            const unsigned par = (pipe.parity >> b) & 1u;
+            const bool got = mbar_wait(pipe.bar + b, par, v.flags);
             pipe.parity ^= 1u << b;
+            all_got = all_got && got;
+            if (tid == 0 && !got) {
+                mbar_drain(pipe.bar + b, par);   // let the late copy land
+                stop = true;
+            }
             float* As = wbuf + b * chunk_floats<TU>();
             float* Ds = As + kPC * kTJ;   // TU / kDB delta blocks of [kPC][kDB]
             const int pc = B - c * kPC;
-            if (pc < kPC) {
-                // rows past the group may hold stale scratch rows: clear those
-                // in the share of the last warp with live rows (the warps after
-                // it skip the chunk)
-                const int pend = min(kPC, (pc + kWarpRows - 1) / kWarpRows * kWarpRows);
+            if (got && warp * kWarpRows < pc) {   // warp-uniform: the warp has live rows
+                if (pc < kPC) {
+                    // this warp's rows past the group may hold stale scratch rows
+                    const int r0 = max(pc, warp * kWarpRows), r1 = (warp + 1) * kWarpRows;
 #pragma unroll
-                for (int h = 0; h < TU / kDB; ++h)
-                    for (int e = tid; e < (pend - pc) * kDB; e += kThreads) Ds[h * kPC * kDB + pc * kDB + e] = 0.f;
-                for (int e = tid; e < (pend - pc) * kTJ; e += kThreads) As[pc * kTJ + e] = 0.f;
-                __syncthreads();
-            }
-            if (warp * kWarpRows < pc) {   // warp-uniform: the warp has live rows
+                    for (int h = 0; h < TU / kDB; ++h)
+                        for (int e = lane; e < (r1 - r0) * kDB; e += 32) Ds[h * kPC * kDB + r0 * kDB + e] = 0.f;
+                    for (int e = lane; e < (r1 - r0) * kTJ; e += 32) As[r0 * kTJ + e] = 0.f;
+                    __syncwarp();
+                }
                 // (the 16-row form unrolls less: its 64 sums leave fewer registers)
 #pragma unroll(TU == kTU ? kWarpRows / 4 : 2)
                 for (int i = 0; i < kWarpRows / 4; ++i) {
@@ -1053,25 +1066,24 @@ __device__ bool weight_phase(const F32View& v, int B, bool fused, bool fold_g, f
                     }
                 }
             }
-            if (__syncthreads_or(!got)) {
-                // a chunk did not arrive in time: issue nothing more and let
-                // every copy already issued land (chunks c + 1 .. c + kNBuf - 1,
-                // and chunk c if thread 0 did not see it complete)
-                if (tid == 0) {
-                    if (!got) mbar_drain(pipe.bar + b, ((pipe.parity >> b) & 1u) ^ 1u);
-                    for (int c2 = c + 1; c2 < c1 && c2 < c + kNBuf; ++c2) {
-                        const int bk = c2 % kNBuf;
-                        mbar_drain(pipe.bar + bk, (pipe.parity >> bk) & 1u);
+            // this warp is done with buffer b; thread 0 refills it once all warps are
+            __syncwarp();
+            if (lane == 0) asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(pipe.ebar + b)) : "memory");
+            if (tid == 0) {
+                const unsigned epar = (pipe.eparity >> b) & 1u;
+                pipe.eparity ^= 1u << b;
+                if (!stop && c + kNBuf < c1) {
+                    if (mbar_wait(pipe.ebar + b, epar, v.flags)) {
+                        asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+                        issue_chunk<TU>(v, pipe, wbuf, l, tb, cb, c + kNBuf, min(kPC, B - (c + kNBuf) * kPC));
+                    } else {
+                        stop = true;
                     }
                 }
-                __syncthreads();
-                return false;
-            }
-            if (tid == 0 && c + kNBuf < c1) {
-                asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-                issue_chunk<TU>(v, pipe, wbuf, l, tb, cb, c + kNBuf, min(kPC, B - (c + kNBuf) * kPC));
             }
         }
+        // a wait ran out: thread 0 has waited for (or drained) every copy it issued
+        if (__syncthreads_or(!all_got || stop)) return false;
         // sum over the 4 pattern lanes (lane bits 4, 3), halving the values at
         // each level: afterwards the lane holds values 0 .. TU - 1 of units
         // ub .. ub + TU / 4 - 1, ub = TU / 2 bit4 + TU / 4 bit3 (each sum is
@@ -1148,16 +1160,21 @@ __device__ void weight_fixup(const F32View& v, int B, bool fold_g) {
     asm volatile("fence.proxy.async.global;" ::: "memory");
 }
 
-// Initialises the weight-phase mbarriers (static shared memory) of a launch.
+// Initialises the weight-phase mbarriers (static shared memory, 2 kNBuf: the
+// full barriers, then the empty ones) of a launch.
 __device__ void pipe_init(ChunkPipe& pipe, uint64_t* bars) {
     if (threadIdx.x == 0) {
         for (int b = 0; b < kNBuf; ++b)
             asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(smem_u32(bars + b)) : "memory");
+        for (int b = 0; b < kNBuf; ++b)
+            asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(bars + kNBuf + b)), "n"(kWarps) : "memory");
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     }
     __syncthreads();
     pipe.bar = bars;
     pipe.parity = 0;
+    pipe.ebar = bars + kNBuf;
+    pipe.eparity = 0;
 }
 
 // Error sum of the group by the first warp of the last CTA: lane-strided
@@ -1245,7 +1262,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 __global__ void __launch_bounds__(kThreads, 1)
     k_accumulate(const __grid_constant__ F32View v, int B, int nparts, float* sse_out) {
     extern __shared__ __align__(128) float smem[];
-    __shared__ __align__(8) uint64_t s_cbar[kNBuf];
+    __shared__ __align__(8) uint64_t s_cbar[2 * kNBuf];
     ChunkPipe pipe;
     pipe_init(pipe, s_cbar);
     reduce_sse(v, nparts, sse_out);
@@ -1271,7 +1288,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             int n_patterns, int minibatch, int n_steps, float* sse_out, int fold_g) {
     extern __shared__ __align__(128) float smem[];
     __shared__ __align__(8) uint64_t s_bar;
-    __shared__ __align__(8) uint64_t s_cbar[kNBuf];
+    __shared__ __align__(8) uint64_t s_cbar[2 * kNBuf];
     // A latched timeout means an earlier launch left the barrier half-way; do
     // nothing until bp_check() has cleared the latch and reset the barrier.
     if (__ldcg(v.flags) & kFlagTimeout) return;
