@@ -267,14 +267,14 @@ def synth_sizes(name):
 # training step (all launches) for the bf16 nets.  Re-measure after any change
 # to these kernels.
 TRAFFIC_PER_PATTERN = {
-    "nettalk60": 1_115_392 / 1024,          # 1.12 MB per launch (one update of 1,024)
-    "nettalk120": 15_406_592 / 16384,       # 61.6 MB per 65,536-pattern launch
+    "nettalk60": 1_116_416 / 1024,          # 1.12 MB per launch (one update of 1,024)
+    "nettalk120": 15_408_128 / 16384,       # 61.6 MB per 65,536-pattern launch
     "wide3": 585_467_136 / 8192,            # 585 MB per step
     "wide4096": 9_221_444_864 / 16384,      # 9.22 GB per step
 }
 # sweep groups of 203-120-26 with a capture of their own (bytes per pattern of one launch);
 # at B = 65,536 the group's scratch rows no longer fit the L2 and make a DRAM round trip
-SWEEP_TRAFFIC_PER_PATTERN = {512: TRAFFIC_PER_PATTERN["nettalk120"], 65536: 594_142_976 / 65536}
+SWEEP_TRAFFIC_PER_PATTERN = {512: TRAFFIC_PER_PATTERN["nettalk120"], 65536: 676_348_928 / 65536}
 
 
 def connections(sizes):
