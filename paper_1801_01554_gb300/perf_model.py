@@ -89,13 +89,13 @@ class GB300Phases:
     pass_us: tuple = ((1, 3.10), (2, 3.43), (4, 4.56), (8, 7.09), (32, 16.3))
     # whole-tile weight phase (8 x 32 tiles, one per CTA): fixed part, then per
     # 512-pattern chunk a fixed and a per-row part
-    weight_fixed_us: float = 1.27
+    weight_fixed_us: float = 1.19
     chunk_fixed_us: float = 0.58
     chunk_rows_us: float = 0.72        # for a full chunk of 512 rows
     # balanced weight phase (16 x 32 tiles, equal runs of chunks per CTA, one
     # more grid barrier and the fix-up): fixed part and per chunk of a run
     balanced_fixed_us: float = 6.66
-    balanced_chunk_us: float = 2.23
+    balanced_chunk_us: float = 2.12
     balanced_min_chunks: int = 24
     chunk_rows: int = 512
     # one-CTA kernel: per group of B patterns
