@@ -268,12 +268,15 @@ bp_status bp_train_epoch_noalloc(const int* layer_sizes, int n_layers, float lr,
 /* Test hook for the failure detection of Section 8 (a processor that stops
  * answering must be noticed, not waited for): float32 nets, checked builds
  * (-DBP_CHECK) only.  Sets the limit of the training kernel's grid-barrier
- * waits to wait_ns nanoseconds (0 restores the default of 2 s) and, if
- * unreachable != 0, moves the count that the next training launch's barriers
- * wait for out of reach, so that its first grid barrier runs out of time: the
- * launch then latches the timeout, every CTA returns with no copy in flight
- * and no update applied, and bp_check reports BP_ETIMEOUT and resets the
- * barrier.  Synchronises the device.  Errors: BP_EINVAL (NULL, a BP_BF16 net),
+ * and weight-phase waits to wait_ns nanoseconds (0 restores the default of
+ * 2 s).  unreachable == 1 moves the count that the next training launch's
+ * barriers wait for out of reach, so that its first grid barrier runs out of
+ * time; unreachable == 2 makes the first chunk copy of each CTA's weight phase
+ * a copy that never comes (its barrier is armed for the bytes, no copy is
+ * issued), so that the chunk waits run out.  Either way the launch latches the timeout,
+ * every CTA returns with every copy it issued landed and no update applied,
+ * and bp_check reports BP_ETIMEOUT and resets the barrier; 0 turns both off.
+ * Synchronises the device.  Errors: BP_EINVAL (NULL, a BP_BF16 net),
  * BP_ESTATE (a library built without BP_CHECK: the hook does nothing there),
  * BP_ECUDA. */
 bp_status bp_debug_wait_test(bp_net* net, unsigned long long wait_ns, int unreachable);

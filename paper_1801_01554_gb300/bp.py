@@ -269,9 +269,10 @@ def bp_train_epoch_noalloc(sizes, lr, momentum, grad_scale, theta, V, X, T, n_pa
 
 
 def bp_debug_wait_test(h, wait_ns, unreachable):
-    """Checked builds only: grid-barrier wait limit (0 = default) and, with
-    unreachable, a first barrier that the next training launch cannot pass."""
-    _check(load().bp_debug_wait_test(h, int(wait_ns), 1 if unreachable else 0))
+    """Checked builds only: grid-barrier and weight-phase wait limit (0 =
+    default); unreachable = 1: a first grid barrier that the next training
+    launch cannot pass; 2: a first weight-phase chunk copy that never comes."""
+    _check(load().bp_debug_wait_test(h, int(wait_ns), int(unreachable)))
 
 
 def bp_last_error() -> str:

@@ -512,7 +512,8 @@ bp_status bp_debug_wait_test(bp_net* net, unsigned long long wait_ns, int unreac
 #ifdef BP_CHECK
     BP_CUDA(cudaDeviceSynchronize(), "bp_debug_wait_test");
     net->view.wait_ns = wait_ns;
-    if (unreachable) {
+    net->view.debug_stall = unreachable == 2 ? 1 : 0;
+    if (unreachable == 1) {
         // barrier k of the next launch waits for bar[0] + k * grid arrivals
         unsigned words[2] = {0, 0};
         BP_CUDA(cudaMemcpy(words, net->bar, sizeof words, cudaMemcpyDeviceToHost), "bp_debug_wait_test");

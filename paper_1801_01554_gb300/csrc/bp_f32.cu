@@ -221,11 +221,12 @@ __device__ __forceinline__ bool mbar_try(uint64_t* bar, unsigned parity) {
 // timeout latches kFlagTimeout and returns false.  The copy it waited for may
 // then still be in flight: the caller issues no more copies and drains
 // (mbar_drain) every copy it issued before the CTA may return.
-__device__ __forceinline__ bool mbar_wait(uint64_t* bar, unsigned parity, int* flags) {
+__device__ __forceinline__ bool mbar_wait(uint64_t* bar, unsigned parity, int* flags,
+                                          unsigned long long limit_ns = kWaitNs) {
     const unsigned long long t0 = global_ns();
     for (unsigned it = 0;; ++it) {
         if (mbar_try(bar, parity)) return true;
-        if ((it & 255u) == 255u && global_ns() - t0 > kWaitNs) {
+        if ((it & 255u) == 255u && global_ns() - t0 > limit_ns) {
             atomicOr(flags, kFlagTimeout);
             return false;
         }
@@ -235,9 +236,9 @@ __device__ __forceinline__ bool mbar_wait(uint64_t* bar, unsigned parity, int* f
 // Second bounded wait for a copy whose first wait ran out, so that its bulk
 // writes land before the CTA exits (shared memory of an exited CTA may belong
 // to the next CTA on that SM).  The error is already latched.
-__device__ __forceinline__ void mbar_drain(uint64_t* bar, unsigned parity) {
+__device__ __forceinline__ void mbar_drain(uint64_t* bar, unsigned parity, unsigned long long limit_ns = kWaitNs) {
     const unsigned long long t0 = global_ns();
-    while (!mbar_try(bar, parity) && global_ns() - t0 < kWaitNs) {
+    while (!mbar_try(bar, parity) && global_ns() - t0 < limit_ns) {
     }
 }
 
@@ -844,15 +845,18 @@ struct ChunkPipe {
 // buffer c % kNBuf: the [rows][kTJ] activation block cb of layer l - 1, then
 // the TU / kDB delta blocks of the tile's units (blocks tb * TU / kDB ..) of
 // layer l, each one contiguous bulk copy from the blocked scratch.  Thread 0 only.
+//   lost: arm the barrier for the chunk's bytes but issue no copy (the checked
+//   build's test hook: a copy that never comes, with nothing in flight)
 template <int TU>
 __device__ __forceinline__ void issue_chunk(const F32View& v, ChunkPipe& pipe, float* wbuf, int l,
-                                            int tb, int cb, int c, int rows) {
+                                            int tb, int cb, int c, int rows, bool lost = false) {
     const int b = c % kNBuf;
     float* buf = wbuf + b * chunk_floats<TU>();
     const unsigned abytes = (unsigned)rows * kTJ * 4, dbytes = (unsigned)rows * kDB * 4;
     asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_u32(pipe.bar + b)),
                  "r"(abytes + (TU / kDB) * dbytes)
                  : "memory");
+    if (lost) return;
     const long long p0 = (long long)c * kPC;
     bulk_load(buf, v.A + v.aoff[l - 1] + (long long)cb * v.cap * kTJ + p0 * kTJ, abytes, pipe.bar + b);
 #pragma unroll
@@ -898,8 +902,12 @@ __device__ __forceinline__ void issue_tile_start(const F32View& v, ChunkPipe& pi
                                                  const Tile& tl, int B, int c0, int c1) {
     asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
     asm volatile("fence.proxy.async.global;" ::: "memory");
+    bool lose_first = false;
+#ifdef BP_CHECK
+    lose_first = v.debug_stall != 0;   // test hook: the first chunk's copy never comes
+#endif
     for (int c = c0; c < c1 && c < c0 + kNBuf; ++c)
-        issue_chunk<TU>(v, pipe, wbuf, tl.l, tl.tb, tl.cb, c, min(kPC, B - c * kPC));
+        issue_chunk<TU>(v, pipe, wbuf, tl.l, tl.tb, tl.cb, c, min(kPC, B - c * kPC), lose_first && c == c0);
 }
 
 // Balanced weight phase for large groups: on tiles of kTUW rows (twice the
@@ -1025,11 +1033,11 @@ __device__ bool weight_phase(const F32View& v, int B, bool fused, bool fold_g, f
         for (int c = c0; c < c1; ++c) {
             const int b = c % kNBuf;
             const unsigned par = (pipe.parity >> b) & 1u;
-            const bool got = mbar_wait(pipe.bar + b, par, v.flags);
+            const bool got = mbar_wait(pipe.bar + b, par, v.flags, wait_limit_ns(v));
             pipe.parity ^= 1u << b;
             all_got = all_got && got;
             if (tid == 0 && !got) {
-                mbar_drain(pipe.bar + b, par);   // let the late copy land
+                mbar_drain(pipe.bar + b, par, wait_limit_ns(v));   // let the late copy land
                 stop = true;
             }
             float* As = wbuf + b * chunk_floats<TU>();
@@ -1073,7 +1081,7 @@ __device__ bool weight_phase(const F32View& v, int B, bool fused, bool fold_g, f
                 const unsigned epar = (pipe.eparity >> b) & 1u;
                 pipe.eparity ^= 1u << b;
                 if (!stop && c + kNBuf < c1) {
-                    if (mbar_wait(pipe.ebar + b, epar, v.flags)) {
+                    if (mbar_wait(pipe.ebar + b, epar, v.flags, wait_limit_ns(v))) {
                         asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
                         issue_chunk<TU>(v, pipe, wbuf, l, tb, cb, c + kNBuf, min(kPC, B - (c + kNBuf) * kPC));
                     } else {

@@ -76,7 +76,8 @@ struct F32View {
     int sig_table;        // 1: table-lookup logistic (Section 4.3) in the forward pass
     float guard;          // > 0: fault guard of Section 8 (|change| > guard is zeroed)
     unsigned* faults;     // changes the guard zeroed (flags[1])
-    unsigned long long wait_ns;   // checked build: grid-barrier wait limit (0: the default 2 s)
+    unsigned long long wait_ns;   // checked build: grid-barrier and weight-phase wait limit (0: the default 2 s)
+    int debug_stall;              // checked build: the weight phase's first chunk never completes (test hook)
 };
 
 // Offsets (floats, each a multiple of 4) of a CTA's pattern buffers for PG

@@ -20,8 +20,8 @@ pytestmark = pytest.mark.gpu
 ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
 
 
-def _run(lib, script="checked_cases.py"):
-    r = subprocess.run([sys.executable, os.path.join(ROOT, "tests", script), lib],
+def _run(lib, script="checked_cases.py", *args):
+    r = subprocess.run([sys.executable, os.path.join(ROOT, "tests", script), lib, *args],
                        capture_output=True, text=True, timeout=600, cwd=ROOT)
     assert r.returncode == 0, r.stderr[-3000:]
     return json.loads(r.stdout.strip().splitlines()[-1])
@@ -48,20 +48,25 @@ def test_checked_build_passes_its_checks_and_matches(checked_lib):
         assert a[k]["agree"] > 0
 
 
-def test_barrier_wait_that_runs_out_is_reported_and_recovered(checked_lib):
-    """Section 8's failure detection without a fault: the first grid barrier of
-    a training launch waits for a count no CTA reaches, with a 1 ms limit.  The
-    launch latches the timeout and stops before any update; bp_check reports
-    BP_ETIMEOUT, clears the latch and resets the barrier; the next epoch on the
-    same net matches the oracle (float32 bar, per layer)."""
+@pytest.mark.parametrize("mode,case", [("barrier", "nettalk120_512"), ("chunk", "nettalk120_512"),
+                                       ("chunk", "nettalk60_12288")])
+def test_wait_that_runs_out_is_reported_and_recovered(checked_lib, mode, case):
+    """Section 8's failure detection without a fault, with a 1 ms limit: either
+    the first grid barrier of a training launch waits for a count no CTA
+    reaches, or the first chunk copy of every CTA's weight phase never comes
+    (whole-tile and balanced weight phases).  The launch latches the timeout
+    and stops before any update; bp_check reports BP_ETIMEOUT, clears the latch
+    and resets the barrier; the next epoch on the same net matches the oracle
+    (float32 bar, per layer)."""
     import numpy as np
     from oracle import bp_oracle as O
     from paper_1801_01554_gb300 import bp, synth
-    r = _run(checked_lib, "timeout_case.py")
+    r = _run(checked_lib, "timeout_case.py", mode, case)
     assert r["status"] == bp.BP_ETIMEOUT
     assert r["weights_unchanged"]
     assert r["seconds"] < 1.0          # the 1 ms limit, not the default 2 s
-    sizes, n, mb = (203, 120, 26), 2048, 512
+    sizes, n, mb = {"nettalk120_512": ((203, 120, 26), 2048, 512),
+                    "nettalk60_12288": ((203, 60, 26), 24576, 12288)}[case]
     X, T = synth.nettalk_patterns(n, seed=71)
     theta = synth.round_to(synth.init_uniform(sizes, -0.3, 0.3, 71), "f32")
     st = O.State(sizes, theta, lr=0.05, momentum=0.9)
