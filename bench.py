@@ -269,8 +269,8 @@ def synth_sizes(name):
 TRAFFIC_PER_PATTERN = {
     "nettalk60": 1_116_416 / 1024,          # 1.12 MB per launch (one update of 1,024)
     "nettalk120": 15_408_128 / 16384,       # 61.6 MB per 65,536-pattern launch
-    "wide3": 585_467_136 / 8192,            # 585 MB per step
-    "wide4096": 9_221_444_864 / 16384,      # 9.22 GB per step
+    "wide3": 586_038_016 / 8192,            # 586 MB per step
+    "wide4096": 9_697_254_656 / 16384,      # 9.70 GB per step (two fp32 partial planes of G)
 }
 # sweep groups of 203-120-26 with a capture of their own (bytes per pattern of one launch);
 # at B = 65,536 the group's scratch rows no longer fit the L2 and make a DRAM round trip

@@ -741,7 +741,9 @@ __device__ __forceinline__ float guard_change(const UpdArgs& a, float g) {
 // Momentum update of Section 6.2.1 over 64 x 64 weight tiles plus the biases:
 // g = sum of partial changes (+ pending G); v = lr*gs*g + m*v; w += v; then the
 // bf16 copy and its transpose.  Mode 1 adds the partial changes into G instead.
-__global__ void __launch_bounds__(256) k_update_bf16(UpdArgs a) {
+// The kernel waits on DRAM latency: three CTAs per SM (80 registers, no spill),
+// and two partial planes' loads issued together, keep more bytes in flight.
+__global__ void __launch_bounds__(256, 3) k_update_bf16(UpdArgs a) {
     if (blockIdx.x == 0 && threadIdx.x == 0 && a.sse_out != nullptr) {
         float s = 0.f;
         for (int k = 0; k < a.n_sse; ++k) s += a.sse_part[k];
@@ -770,7 +772,7 @@ __global__ void __launch_bounds__(256) k_update_bf16(UpdArgs a) {
             const int j0 = rb * kUT + (w >> 1) * 16 + (lane >> 3) * 4;
             if (i < u.n_in && j0 < u.n_out) {
                 const float4 z = make_float4(0.f, 0.f, 0.f, 0.f);
-                float4 gs[4], w4[4], v4[4], gp4[4];
+                float4 gs[4], w4[4], v4[4];
                 const size_t e0 = (size_t)j0 * u.n_in + i;
                 const float* th = a.theta + u.woff + e0;
                 float* vv = a.V + u.woff + e0;
@@ -779,16 +781,33 @@ __global__ void __launch_bounds__(256) k_update_bf16(UpdArgs a) {
                 for (int r = 0; r < 4; ++r) {
                     gs[r] = z;
                     v4[r] = z;
-                    gp4[r] = z;
                     w4[r] = *reinterpret_cast<const float4*>(th + (size_t)r * u.n_in);
-                    if (a.mode == 0) {
-                        v4[r] = *reinterpret_cast<const float4*>(vv + (size_t)r * u.n_in);
-                        if (a.fold_g) gp4[r] = *reinterpret_cast<const float4*>(gg + (size_t)r * u.n_in);
-                    }
+                    if (a.mode == 0) v4[r] = *reinterpret_cast<const float4*>(vv + (size_t)r * u.n_in);
                 }
                 if (a.mode != 2) {
                     const size_t plane = (size_t)u.n_out * u.n_in;
-                    for (int s = 0; s < u.splits; ++s) {
+                    int s0 = 0;
+                    for (; s0 + 2 <= u.splits; s0 += 2) {
+                        const float* gp = u.gpart + s0 * plane + e0;
+                        float4 p0[4], p1[4];
+#pragma unroll
+                        for (int r = 0; r < 4; ++r) {
+                            p0[r] = __ldcs(reinterpret_cast<const float4*>(gp + (size_t)r * u.n_in));
+                            p1[r] = __ldcs(reinterpret_cast<const float4*>(gp + plane + (size_t)r * u.n_in));
+                        }
+#pragma unroll
+                        for (int r = 0; r < 4; ++r) {
+                            gs[r].x += p0[r].x;
+                            gs[r].y += p0[r].y;
+                            gs[r].z += p0[r].z;
+                            gs[r].w += p0[r].w;
+                            gs[r].x += p1[r].x;
+                            gs[r].y += p1[r].y;
+                            gs[r].z += p1[r].z;
+                            gs[r].w += p1[r].w;
+                        }
+                    }
+                    for (int s = s0; s < u.splits; ++s) {
                         const float* gp = u.gpart + s * plane + e0;
 #pragma unroll
                         for (int r = 0; r < 4; ++r) {
@@ -811,10 +830,11 @@ __global__ void __launch_bounds__(256) k_update_bf16(UpdArgs a) {
                         g4.w += gs[r].w;
                         *reinterpret_cast<float4*>(gg + o) = g4;
                     } else if (a.mode == 0) {
+                        const float4 gp4 = a.fold_g ? *reinterpret_cast<const float4*>(gg + o) : z;
                         float* wc = &w4[r].x;
                         float* vc = &v4[r].x;
                         const float* gc = &gs[r].x;
-                        const float* pc = &gp4[r].x;
+                        const float* pc = &gp4.x;
 #pragma unroll
                         for (int c = 0; c < 4; ++c) {
                             const float vel = a.lr_gs * guard_change(a, gc[c] + pc[c]) + a.momentum * vc[c];
