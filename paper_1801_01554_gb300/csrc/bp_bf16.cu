@@ -959,6 +959,10 @@ struct Bf16Net {
     float* bpart[BP_MAX_SIZES] = {nullptr}; // [mtiles(cap), n_l]
     float* sse_part = nullptr;              // [mtiles(cap) * tiles along n_L]
     int n_sse_cap = 0;
+    // X^T runs on a stream of the net's own, forked from and joined back into
+    // the caller's stream, beside the hidden-delta GEMMs
+    cudaStream_t side = nullptr;
+    cudaEvent_t fork = nullptr, join = nullptr;
     std::vector<void*> allocs;
 };
 
@@ -1066,19 +1070,30 @@ cudaError_t run_forward(Bf16Net* b, const bf16* X, int B, const bf16* T, bf16* Y
 // and the activations must already be in scratch).
 cudaError_t run_backward(Bf16Net* b, const bf16* X, int B, cudaStream_t s) {
     const int L = b->L;
-    // X^T for the first layer's pooled change
+    // X^T for the first layer's pooled change, on the side stream: it reads only
+    // X, so it overlaps the hidden-delta GEMMs (one 8.4 KB transpose block fits
+    // beside a GEMM CTA on an SM).  The fork orders it after everything already
+    // on s, the previous group's read of the same buffer included; the join
+    // orders the pooled-change GEMMs after it.
     {
+        cudaError_t e = cudaEventRecord(b->fork, s);
+        if (e == cudaSuccess) e = cudaStreamWaitEvent(b->side, b->fork, 0);
+        if (e != cudaSuccess) return e;
         dim3 grid(ceil_div(b->n[0], 64), ceil_div(B, 64));
-        k_transpose<<<grid, 256, 0, s>>>(X, B, b->n[0], b->n[0], b->actT[0], b->cap_pad);
-        cudaError_t e = cudaGetLastError();
+        k_transpose<<<grid, 256, 0, b->side>>>(X, B, b->n[0], b->n[0], b->actT[0], b->cap_pad);
+        e = cudaGetLastError();
+        if (e == cudaSuccess) e = cudaEventRecord(b->join, b->side);
         if (e != cudaSuccess) return e;
     }
-    for (int l = L; l >= 2; --l) {
+    cudaError_t e_dx = cudaSuccess;
+    for (int l = L; l >= 2 && e_dx == cudaSuccess; --l) {
         // delta_{l-1} = (delta_l W_l) * a (1 - a):  A = delta_l [B, n_l], B-operand = W_l^T
         CUtensorMap ma, mb;
         if (!make_map(&ma, b->dlt[l], B, b->n[l], b->n[l], BM) ||
-            !make_map(&mb, b->wt[l], b->n[l - 1], b->n[l], b->n[l], kBN))
-            return cudaErrorInvalidValue;
+            !make_map(&mb, b->wt[l], b->n[l - 1], b->n[l], b->n[l], kBN)) {
+            e_dx = cudaErrorInvalidValue;
+            break;
+        }
         GemmArgs g = blank_args();
         g.M = B;
         g.N = b->n[l - 1];
@@ -1090,9 +1105,12 @@ cudaError_t run_backward(Bf16Net* b, const bf16* X, int B, cudaStream_t s) {
         g.aux = b->act[l - 1];
         g.ld_aux = b->n[l - 1];
         g.bias_part = b->bpart[l - 1];
-        cudaError_t e = launch_gemm<MODE_DX>(b, ma, mb, g, s);
-        if (e != cudaSuccess) return e;
+        e_dx = launch_gemm<MODE_DX>(b, ma, mb, g, s);
     }
+    // joined on every path, so that a stream capture on s stays whole
+    const cudaError_t e_join = cudaStreamWaitEvent(s, b->join, 0);
+    if (e_dx != cudaSuccess) return e_dx;
+    if (e_join != cudaSuccess) return e_join;
     for (int l = 1; l <= L; ++l) {
         // G_l = delta_l^T A_{l-1}: A = delta_l^T [n_l, B], B-operand = A_{l-1}^T [n_{l-1}, B]
         CUtensorMap ma, mb;
@@ -1240,12 +1258,23 @@ bp_status bf16_create(const int* n, int L, int max_batch, int num_sms, float* th
         bf16_destroy(b);
         return BP_ENOMEM;
     }
+    if (cudaStreamCreateWithFlags(&b->side, cudaStreamNonBlocking) != cudaSuccess ||
+        cudaEventCreateWithFlags(&b->fork, cudaEventDisableTiming) != cudaSuccess ||
+        cudaEventCreateWithFlags(&b->join, cudaEventDisableTiming) != cudaSuccess) {
+        g_msg = "could not create the bfloat16 path's side stream and events";
+        bf16_destroy(b);
+        return BP_ECUDA;
+    }
     *out = b;
     return BP_OK;
 }
 
 void bf16_destroy(Bf16Net* b) {
     if (b == nullptr) return;
+    if (b->side) cudaStreamSynchronize(b->side);
+    if (b->fork) cudaEventDestroy(b->fork);
+    if (b->join) cudaEventDestroy(b->join);
+    if (b->side) cudaStreamDestroy(b->side);
     for (void* p : b->allocs) cudaFree(p);
     delete b;
 }
