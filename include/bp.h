@@ -35,6 +35,10 @@
  *   - `stream` is a cudaStream_t passed as void* (NULL = legacy default stream).
  *     Compute entry points are asynchronous with respect to the host; the
  *     device buffers they read must stay valid until the stream reaches them.
+ *     A BP_BF16 net's backward pass forks part of its work (the input
+ *     transpose) onto a stream of the net's own and joins it back into
+ *     `stream` before the call's next dependent kernel, so that the call's
+ *     work is ordered on `stream` as a whole (stream capture included).
  *   - A net must not be used from two host threads at once.
  *   - Every call returns a bp_status; on failure bp_last_error() holds a
  *     message for the calling thread.  Argument errors are detected before any
