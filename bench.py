@@ -265,12 +265,11 @@ def synth_sizes(name):
 # for the float32 nets (one epoch; 203-120-26 captured on a 16,384-pattern epoch
 # and scaled by patterns, as its traffic is the inputs read once), the whole
 # training step (all launches) for the bf16 nets.  Re-measure after any change
-# to these kernels.
+# to these kernels; a workload whose kernels changed since its capture has none
+# (the bf16 nets: the update kernel's bias part changed after their capture).
 TRAFFIC_PER_PATTERN = {
     "nettalk60": 1_116_416 / 1024,          # 1.12 MB per launch (one update of 1,024)
     "nettalk120": 15_408_128 / 16384,       # 61.6 MB per 65,536-pattern launch
-    "wide3": 586_038_016 / 8192,            # 586 MB per step
-    "wide4096": 9_697_254_656 / 16384,      # 9.70 GB per step (two fp32 partial planes of G)
 }
 # sweep groups of 203-120-26 with a capture of their own (bytes per pattern of one launch);
 # at B = 65,536 the group's scratch rows no longer fit the L2 and make a DRAM round trip

@@ -864,13 +864,19 @@ __global__ void __launch_bounds__(256, 3) k_update_bf16(UpdArgs a) {
                     }
                 }
             }
-        } else if (cb == 0) {
-            // biases of this layer
-            for (int j = threadIdx.x; j < u.n_out; j += 256) {
+        } else {
+            // biases of this layer, spread over the `cols` tiles of the bias row (one
+            // tile with the rest idle left a long tail of dependent partial-sum loads);
+            // each bias sums its row-block partials in order, loads issued 16 ahead
+            const int per = (u.n_out + cols - 1) / cols;
+            const int j_hi = min(u.n_out, (cb + 1) * per);
+            for (int j = cb * per + threadIdx.x; j < j_hi; j += 256) {
                 const long long idx = u.boff + j;
                 float gsum = 0.f;
-                if (a.mode != 2)
+                if (a.mode != 2) {
+#pragma unroll 16
                     for (int mt = 0; mt < u.mtiles; ++mt) gsum += u.bias_part[(size_t)mt * u.n_out + j];
+                }
                 if (a.mode == 1) {
                     a.G[idx] += gsum;
                 } else if (a.mode == 0) {
